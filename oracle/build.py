@@ -1,0 +1,26 @@
+"""Compile the C oracle into oracle/liboracle.so with the host C compiler.
+
+Test infrastructure: builds the checker only. Plain C, no architecture flags,
+so the same source builds on x86_64 and aarch64 hosts.
+"""
+import os
+import subprocess
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+SRC = os.path.join(HERE, "dkv_oracle.c")
+LIB = os.path.join(HERE, "liboracle.so")
+
+
+def build(force: bool = False) -> str:
+    if not force and os.path.exists(LIB) and os.path.getmtime(LIB) >= os.path.getmtime(SRC):
+        return LIB
+    cc = os.environ.get("CC", "gcc")
+    tmp = LIB + ".tmp"
+    subprocess.check_call([cc, "-O2", "-std=c11", "-fPIC", "-shared", "-Wall", "-Wextra",
+                           "-o", tmp, SRC, "-lm"])
+    os.replace(tmp, LIB)
+    return LIB
+
+
+if __name__ == "__main__":
+    print(build(force=True))

@@ -1,0 +1,217 @@
+"""Seeded synthetic inputs for the Distance-KV decode path.
+
+This module only draws inputs: retention patterns M, context lengths, and the
+bf16 K/V/q tensors. It holds none of the method's arithmetic (no distance bins,
+no retention mask, no packing, no attention), so both the CUDA path and the CPU
+oracle can be fed from it without sharing any of the computation.
+
+The workloads stand in for the paper's efficiency setting (Sec. 4.3, App. C:
+Llama-3.1-8B and Qwen2.5-7B caches up to 128K context on one GPU). No model
+weights or datasets are used: K, V, q are N(0, 1) bf16 draws, and patterns come
+from seeded generators shaped like the learned ones (Sec. 4.5: near-heavy, a
+far rise for some heads, partial heads).
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field, replace
+
+import numpy as np
+
+SINK = 128      # Sec. 3.4: first 128 context positions always kept
+RECENT = 1024   # Sec. 3.4: most recent 1,024 context positions always kept
+
+
+@dataclass(frozen=True)
+class Workload:
+    """One benchmark/test workload: model head geometry, context mix, pattern recipe."""
+    name: str
+    L: int
+    H: int
+    Hkv: int
+    T: int                      # maximum (and, unless ragged, every) context length
+    B: int
+    D: int                      # distance bins of the pattern
+    W: int                      # bin width in tokens (a property of the pattern)
+    pattern: str                # "bernoulli" | "profile"
+    rate: float                 # bernoulli: P(M=1); profile: fraction of union bins kept
+    physical_target: float | None = None  # profile: choose K_U for this overall physical retention
+    ragged: tuple | None = None  # (lo, hi): per-sequence lengths uniform in [lo, hi]
+    outlier_frac: float = 0.0   # fraction of key rows scaled by 8 (exact in bf16)
+    seed: int = 0
+    steps: int = 256
+    head_dim: int = 128
+    sink: int = SINK
+    recent: int = RECENT
+    extra: dict = field(default_factory=dict)
+
+    @property
+    def G(self) -> int:
+        return self.H // self.Hkv
+
+    def with_(self, **kw) -> "Workload":
+        return replace(self, **kw)
+
+
+def _w(T, D):
+    return (T - SINK - RECENT) // D
+
+
+# The five benchmark workloads (Llama-3.1-8B: 32 layers, 32 q-heads, 8 KV heads;
+# Qwen2.5-7B: 28 layers, 28 q-heads, 4 KV heads; head_dim 128 for both).
+WORKLOADS = {
+    "llama8b-1layer-4k": Workload("llama8b-1layer-4k", L=1, H=32, Hkv=8, T=4096, B=1, D=32,
+                                  W=_w(4096, 32), pattern="bernoulli", rate=0.35, seed=1),
+    "llama8b-32k": Workload("llama8b-32k", L=32, H=32, Hkv=8, T=32768, B=1, D=64,
+                            W=_w(32768, 64), pattern="profile", rate=0.35, seed=2),
+    "llama8b-128k": Workload("llama8b-128k", L=32, H=32, Hkv=8, T=131072, B=1, D=128,
+                             W=_w(131072, 128), pattern="profile", rate=0.346,
+                             physical_target=0.346, outlier_frac=0.01, seed=3),
+    "llama8b-b16-ragged": Workload("llama8b-b16-ragged", L=32, H=32, Hkv=8, T=65536, B=16, D=64,
+                                   W=_w(65536, 64), pattern="profile", rate=0.25,
+                                   ragged=(8192, 65536), seed=4),
+    "qwen7b-64k-b4-r20": Workload("qwen7b-64k-b4-r20", L=28, H=28, Hkv=4, T=65536, B=4, D=64,
+                                  W=_w(65536, 64), pattern="profile", rate=0.20, seed=5),
+    "qwen7b-64k-b4-r35": Workload("qwen7b-64k-b4-r35", L=28, H=28, Hkv=4, T=65536, B=4, D=64,
+                                  W=_w(65536, 64), pattern="profile", rate=0.35, seed=5),
+    "qwen7b-64k-b4-r50": Workload("qwen7b-64k-b4-r50", L=28, H=28, Hkv=4, T=65536, B=4, D=64,
+                                  W=_w(65536, 64), pattern="profile", rate=0.50, seed=5),
+}
+
+
+def context_lengths(wl: Workload) -> np.ndarray:
+    """Per-sequence context lengths T_c[b] (int32)."""
+    if wl.ragged is None:
+        return np.full(wl.B, wl.T, np.int32)
+    rng = np.random.default_rng([wl.seed, 11])
+    lo, hi = wl.ragged
+    return rng.integers(lo, hi + 1, size=wl.B, dtype=np.int64).astype(np.int32)
+
+
+def topk_mask(scores: np.ndarray, k: int) -> np.ndarray:
+    """Global Top-K of a score tensor (Eq. 3 / App. A.3 shape): the k largest
+    entries become 1. Ties go to the lower flat index (stable order)."""
+    flat = scores.reshape(-1)
+    k = int(max(0, min(k, flat.size)))
+    order = np.argsort(-flat, kind="stable")
+    out = np.zeros(flat.size, np.uint8)
+    out[order[:k]] = 1
+    return out.reshape(scores.shape)
+
+
+def round_half_up(x: float) -> int:
+    """round() of App. A.3 read as floor(x + 0.5)."""
+    return int(np.floor(x + 0.5))
+
+
+def bernoulli_pattern(wl: Workload, rng: np.random.Generator) -> np.ndarray:
+    """Per (layer, q-head, bin) Bernoulli(rate), with the nearest bin (d=0) always on."""
+    M = (rng.random((wl.L, wl.H, wl.D)) < wl.rate).astype(np.uint8)
+    if wl.D > 0:
+        M[:, :, 0] = 1
+    return M
+
+
+def union_bins_target(wl: Workload) -> int:
+    """Number K_U of (layer, KV head, bin) entries the profile generator keeps."""
+    if wl.physical_target is not None:
+        # Overall physical retention r of a T-token context: kept rows per head
+        # = S + R + K_U * W / (L * Hkv) = r * T.
+        per_head_bins = (wl.physical_target * wl.T - wl.sink - wl.recent) / wl.W
+        return round_half_up(per_head_bins * wl.L * wl.Hkv)
+    return round_half_up(wl.rate * wl.L * wl.Hkv * wl.D)
+
+
+def profile_pattern(wl: Workload, rng: np.random.Generator) -> np.ndarray:
+    """Near/far retention profile per (layer, KV head), exact union budget,
+    then a random non-empty subset of the group's q-heads per kept bin.
+
+    score_d = w (1 - x_d) + (1 - w) x_d + 0.25 U(0,1), x_d = d / (D - 1),
+    w ~ Beta(2, 2) per (layer, KV head). A global Top-K keeps K_U union entries.
+    Each kept union bin is given to each q-head of the group with probability
+    1/2, redrawn until at least one q-head has it, so the GQA union of M is
+    exactly the selected set.
+    """
+    L, Hkv, D, G = wl.L, wl.Hkv, wl.D, wl.G
+    w = rng.beta(2.0, 2.0, size=(L, Hkv, 1))
+    x = (np.arange(D) / max(D - 1, 1))[None, None, :]
+    score = w * (1.0 - x) + (1.0 - w) * x + 0.25 * rng.random((L, Hkv, D))
+    U = topk_mask(score, union_bins_target(wl))
+    M = np.zeros((L, Hkv, G, D), np.uint8)
+    sel = np.argwhere(U == 1)
+    for (l, g, d) in sel:
+        while True:
+            pick = rng.random(G) < 0.5
+            if pick.any():
+                break
+        M[l, g, :, d] = pick
+    return M.reshape(L, Hkv * G, D)
+
+
+def make_pattern(wl: Workload) -> np.ndarray:
+    """The workload's retention pattern M in {0,1}^{L x H x D} (uint8)."""
+    rng = np.random.default_rng([wl.seed, 7])
+    if wl.pattern == "bernoulli":
+        return bernoulli_pattern(wl, rng)
+    if wl.pattern == "profile":
+        return profile_pattern(wl, rng)
+    if wl.pattern == "ones":
+        return np.ones((wl.L, wl.H, wl.D), np.uint8)
+    if wl.pattern == "zeros":
+        return np.zeros((wl.L, wl.H, wl.D), np.uint8)
+    raise ValueError(f"unknown pattern recipe {wl.pattern!r}")
+
+
+def dense_kv(wl: Workload, T_stride: int | None = None, device="cpu", layer_chunk: int = 1):
+    """Dense post-RoPE caches K, V, bf16 [L][B][Hkv][T_stride][head_dim] ~ N(0,1).
+
+    Drawn with a torch generator seeded from the workload, K then V, one layer at
+    a time (so the device never holds an fp32 copy of a whole cache). A fraction
+    `outlier_frac` of key rows (Bernoulli per (layer, b, KV head, position)) is
+    multiplied by 8, which is exact in bf16. Rows past a sequence's length are
+    drawn as well; the path never reads them.
+    """
+    import torch
+    T_stride = T_stride or wl.T
+    shape = (wl.L, wl.B, wl.Hkv, T_stride, wl.head_dim)
+    gen = torch.Generator(device=device)
+    gen.manual_seed(wl.seed * 1000 + 17)
+    K = torch.empty(shape, dtype=torch.bfloat16, device=device)
+    V = torch.empty(shape, dtype=torch.bfloat16, device=device)
+    for t in (K, V):
+        for l0 in range(0, wl.L, layer_chunk):
+            l1 = min(wl.L, l0 + layer_chunk)
+            t[l0:l1].copy_(torch.randn((l1 - l0,) + shape[1:], generator=gen, device=device,
+                                       dtype=torch.float32).to(torch.bfloat16))
+    if wl.outlier_frac > 0:
+        for l in range(wl.L):
+            hit = torch.rand(shape[1:4], generator=gen, device=device) < wl.outlier_frac
+            K[l][hit] = K[l][hit] * 8
+    return K, V
+
+
+def decode_inputs(wl: Workload, steps: int, device="cpu", seed_offset: int = 0):
+    """Per-step decode inputs, bf16 ~ N(0,1):
+    q [steps][L][B][H][hd], k_new and v_new [steps][L][B][Hkv][hd]."""
+    import torch
+    gen = torch.Generator(device=device)
+    gen.manual_seed(wl.seed * 1000 + 29 + seed_offset)
+    hd = wl.head_dim
+
+    def draw(*shape):
+        return torch.randn(shape, generator=gen, device=device,
+                           dtype=torch.float32).to(torch.bfloat16)
+    q = draw(steps, wl.L, wl.B, wl.H, hd)
+    k_new = draw(steps, wl.L, wl.B, wl.Hkv, hd)
+    v_new = draw(steps, wl.L, wl.B, wl.Hkv, hd)
+    return q, k_new, v_new
+
+
+def bf16_bits(t) -> np.ndarray:
+    """Raw bf16 bit patterns of a (CPU or CUDA) torch bf16 tensor as uint16."""
+    import torch
+    return t.detach().to("cpu").contiguous().view(torch.int16).numpy().view(np.uint16)
+
+
+__all__ = ["Workload", "WORKLOADS", "SINK", "RECENT", "context_lengths", "make_pattern",
+           "topk_mask", "round_half_up", "union_bins_target", "dense_kv", "decode_inputs",
+           "bf16_bits"]
