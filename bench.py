@@ -1,0 +1,530 @@
+"""Benchmark of the Distance-KV decode hot path on one GB300 (per process).
+
+A step is one decode step of the whole model: for every layer, the split-K
+partial pass (which also appends the step's key/value to the packed cache) and
+the combine pass, then dkv_advance -- replayed as one CUDA graph. Before the
+timed steps the path runs its one-shot part once per context: the pattern map
+and the prune-and-pack (timed separately and reported as compaction GB/s).
+
+Default workload: Llama-3.1-8B-shaped cache (32 layers, 32 q-heads, 8 KV heads,
+head_dim 128), batch 1, 131,072-token context, 34.6 % physical retention,
+1 % outlier keys, synthetic N(0,1) bf16 K/V/q.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl dkv|reference]
+
+--impl reference times the CPU oracle on the same workload (bounded sample of
+the heads of each step, scaled to a full step). Under torchrun every rank runs
+its own replica (the path does not exchange data between GPUs); the timing is
+the max over ranks and rank 0 prints one JSON line.
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2609_32663_gb300 import inputs as I  # noqa: E402
+
+METRIC = "compacted decode-attention us/step (Llama-3.1-8B KV shape, 131072 ctx, 34.6% retention)"
+UNIT = "us/step"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=256)
+    ap.add_argument("--warmup", type=int, default=8)
+    ap.add_argument("--impl", default="dkv", choices=["dkv", "reference"])
+    ap.add_argument("--workload", default="llama8b-128k", choices=sorted(I.WORKLOADS))
+    ap.add_argument("--no-dense", action="store_true", help="skip the dense-cache baseline")
+    ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
+    ap.add_argument("--cpu-layers", type=int, default=2, help="layers of one step the CPU oracle times")
+    ap.add_argument("--profile", action="store_true", help="few steps, no baselines (for ncu)")
+    return ap.parse_args()
+
+
+# ---------------------------------------------------------------- distributed plumbing
+class Dist:
+    def __init__(self, n):
+        self.world = int(os.environ.get("WORLD_SIZE", "1"))
+        self.rank = int(os.environ.get("RANK", "0"))
+        self.local = int(os.environ.get("LOCAL_RANK", "0"))
+        self.pg = None
+        if self.world > 1:
+            import torch
+            import torch.distributed as dist
+            backend = "nccl" if torch.cuda.is_available() else "gloo"
+            dist.init_process_group(backend)
+            self.pg = dist
+
+    def barrier(self):
+        if self.pg:
+            self.pg.barrier()
+
+    def max(self, x):
+        if not self.pg:
+            return x
+        import torch
+        dev = "cuda" if torch.cuda.is_available() else "cpu"
+        t = torch.tensor([float(x)], dtype=torch.float64, device=dev)
+        self.pg.all_reduce(t, op=self.pg.ReduceOp.MAX)
+        return float(t.item())
+
+    def close(self):
+        if self.pg:
+            self.pg.destroy_process_group()
+
+
+# ---------------------------------------------------------------- clocks
+class Clocks:
+    """nvidia-smi sampler over the timed region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.idx = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, smax, reasons, power = [], None, set(), []
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax = float(f[2])
+                power.append(float(f[3]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": smax,
+                "reasons": sorted(reasons), "samples": len(sm),
+                "power_w_max": max(power) if power else None}
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except (OSError, ValueError):
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}, "fallback"
+
+
+# ---------------------------------------------------------------- workload set-up
+def setup(wl, dev, reserve):
+    import torch
+
+    import paper_2609_32663_gb300.dkv as dkv
+    M = I.make_pattern(wl)
+    Tc = I.context_lengths(wl)
+    shape = dkv.Shape(L=wl.L, H=wl.H, H_kv=wl.Hkv, D=wl.D, sink=wl.sink, recent=wl.recent, bin_width=wl.W)
+    T_stride = int(Tc.max()) + reserve  # room for the dense baseline's appended tokens
+    K, V = I.dense_kv(wl.with_(T=T_stride), device=dev)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    plan = dkv.dkv_map_pattern(M, Tc, shape, reserve_rows=reserve)
+    map_ms = (time.perf_counter() - t0) * 1e3
+    info = dkv.dkv_plan_query(plan)
+    Kc = torch.empty((info.total_rows, wl.head_dim), dtype=torch.bfloat16, device=dev)
+    Vc = torch.empty_like(Kc)
+    return dict(M=M, Tc=Tc, shape=shape, T_stride=T_stride, K=K, V=V, plan=plan, info=info, Kc=Kc, Vc=Vc,
+                map_ms=map_ms)
+
+
+def time_compaction(env, reps=10):
+    import torch
+
+    import paper_2609_32663_gb300.dkv as dkv
+    st = torch.cuda.current_stream()
+    times = []
+    for i in range(reps + 2):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(st)
+        dkv.dkv_compact(env["plan"], env["K"], env["V"], env["Kc"], env["Vc"], T_stride=env["T_stride"])
+        e1.record(st)
+        e1.synchronize()
+        if i >= 2:
+            times.append(e0.elapsed_time(e1) * 1e-3)
+    t = statistics.median(times)
+    kept = env["info"].kept_rows
+    algo = kept * (2 * 256 * 2 + 4)  # read K,V rows + write K,V rows + read the 4-byte index
+    return {"gbs": algo / t / 1e9, "ms": t * 1e3, "algorithmic_bytes": algo, "reps": reps}
+
+
+def step_bytes(wl, Tc_rows_per_layer, with_new=True):
+    """Algorithmic bytes of one decode step: retained K/V rows (with appended
+    tokens) + q read + o written + the new K/V row written."""
+    kv = Tc_rows_per_layer * 2 * 256
+    q = wl.B * wl.H * wl.head_dim * 2
+    o = wl.B * wl.H * wl.head_dim * 4
+    new = 2 * wl.B * wl.Hkv * 256 if with_new else 0
+    return kv + q + o + new
+
+
+class DecodeRunner:
+    """One decode step over all layers as a CUDA graph (per-layer partial +
+    combine, then dkv_advance), or the same launches eagerly with per-launch events."""
+
+    def __init__(self, wl, plan, Kc, Vc, dev, seed_offset=0):
+        import torch
+
+        import paper_2609_32663_gb300.dkv as dkv
+        self.dkv, self.torch = dkv, torch
+        self.wl, self.plan, self.Kc, self.Vc = wl, plan, Kc, Vc
+        q, kn, vn = I.decode_inputs(wl, 1, device=dev, seed_offset=seed_offset)
+        self.q, self.kn, self.vn = q[0].contiguous(), kn[0].contiguous(), vn[0].contiguous()
+        self.n_app = torch.zeros(wl.B, dtype=torch.int32, device=dev)
+        self.out = torch.empty((wl.L, wl.B, wl.H, wl.head_dim), dtype=torch.float32, device=dev)
+        self.graph = None
+
+    def launch_step(self):
+        d = self.dkv
+        for layer in range(self.wl.L):
+            d.dkv_decode_partial(self.plan, layer, self.q[layer], self.kn[layer], self.vn[layer], self.n_app,
+                                 self.Kc, self.Vc)
+            d.dkv_decode_combine(self.plan, layer, self.n_app, True, self.out[layer])
+        d.dkv_advance(self.plan, self.n_app)
+
+    def capture(self):
+        torch = self.torch
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            self.launch_step()  # warm the launch path outside capture
+        torch.cuda.current_stream().wait_stream(s)
+        torch.cuda.synchronize()
+        self.n_app.zero_()
+        self.graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(self.graph):
+            self.launch_step()
+        torch.cuda.synchronize()
+        self.n_app.zero_()
+
+    def replay(self):
+        self.graph.replay()
+
+    def timed_partials(self, steps):
+        """Eager steps with CUDA events around every partial launch: mean duration."""
+        torch, d = self.torch, self.dkv
+        st = torch.cuda.current_stream()
+        durs = []
+        for _ in range(steps):
+            evs = []
+            for layer in range(self.wl.L):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(st)
+                d.dkv_decode_partial(self.plan, layer, self.q[layer], self.kn[layer], self.vn[layer], self.n_app,
+                                     self.Kc, self.Vc)
+                e1.record(st)
+                d.dkv_decode_combine(self.plan, layer, self.n_app, True, self.out[layer])
+                evs.append((e0, e1))
+            d.dkv_advance(self.plan, self.n_app)
+            torch.cuda.synchronize()
+            durs.extend(e0.elapsed_time(e1) * 1e-3 for e0, e1 in evs)
+        return statistics.mean(durs), len(durs)
+
+
+def time_graph(runner, steps, warmup, dist, clocks=None):
+    import torch
+    for _ in range(warmup):
+        runner.replay()
+    torch.cuda.synchronize()
+    dist.barrier()
+    torch.cuda.synchronize()
+    if clocks:
+        clocks.start()
+        time.sleep(0.3)
+    st = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(st)
+    for _ in range(steps):
+        runner.replay()
+    e1.record(st)
+    e1.synchronize()
+    torch.cuda.synchronize()
+    clk = clocks.stop() if clocks else None
+    dist.barrier()
+    return e0.elapsed_time(e1) * 1e-3 / steps, clk
+
+
+def run_e2e(wl, plan, Kc, Vc, dev, steps, warmup):
+    """Same step through the public API with host buffers: every step copies its
+    q, k_new, v_new from pinned host memory and reads all layers' outputs back."""
+    import torch
+
+    import paper_2609_32663_gb300.dkv as dkv
+    q, kn, vn = I.decode_inputs(wl, 1, seed_offset=7)
+    hq, hk, hv = q[0].pin_memory(), kn[0].pin_memory(), vn[0].pin_memory()
+    hout = torch.empty((wl.L, wl.B, wl.H, wl.head_dim), dtype=torch.float32).pin_memory()
+    dq, dk, dv = torch.empty_like(hq, device=dev), torch.empty_like(hk, device=dev), torch.empty_like(hv, device=dev)
+    out = torch.empty((wl.L, wl.B, wl.H, wl.head_dim), dtype=torch.float32, device=dev)
+    n_app = torch.zeros(wl.B, dtype=torch.int32, device=dev)
+
+    def step():
+        dq.copy_(hq, non_blocking=True)
+        dk.copy_(hk, non_blocking=True)
+        dv.copy_(hv, non_blocking=True)
+        for layer in range(wl.L):
+            dkv.dkv_decode_attn(plan, layer, dq[layer], dk[layer], dv[layer], n_app, Kc, Vc, out[layer])
+        dkv.dkv_advance(plan, n_app)
+        hout.copy_(out, non_blocking=True)
+
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        step()
+    torch.cuda.current_stream().wait_stream(s)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        step()
+    for _ in range(warmup):
+        g.replay()
+    torch.cuda.synchronize()
+    st = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(st)
+    for _ in range(steps):
+        g.replay()
+    e1.record(st)
+    e1.synchronize()
+    t = e0.elapsed_time(e1) * 1e-3 / steps
+    bi = hq.numel() * 2 + hk.numel() * 2 + hv.numel() * 2
+    bo = hout.numel() * 4
+    return t, bi, bo
+
+
+def cpu_oracle_step(wl, env, layers, dev):
+    """CPU oracle (single thread, fp64) on `layers` layers of one decode step over
+    the packed cache built on the GPU; returns seconds per full step (scaled by L)."""
+    import torch
+
+    import oracle as O
+    import paper_2609_32663_gb300.dkv as dkv
+    ln, off, ioff, idx = dkv.dkv_plan_read(env["plan"])
+    NHl = wl.B * wl.Hkv
+    q, _, _ = I.decode_inputs(wl, 1, seed_offset=3)
+    total = 0.0
+    rows = 0
+    for layer in range(layers):
+        lo, hi = int(off[layer * NHl]), int(off[(layer + 1) * NHl])
+        Kh = I.bf16_bits(env["Kc"][lo:hi])
+        Vh = I.bf16_bits(env["Vc"][lo:hi])
+        m = O.Mapping(ln, off - lo, ioff, idx)
+        qb = I.bf16_bits(q[0, layer])
+        t0 = time.perf_counter()
+        O.decode(m, layer, wl.B, wl.H, wl.Hkv, qb, Kh, Vh)
+        total += time.perf_counter() - t0
+        rows += int(ln[layer * NHl:(layer + 1) * NHl].sum())
+    return total / layers * wl.L, rows
+
+
+def cpu_model():
+    try:
+        with open("/proc/cpuinfo") as f:
+            for ln in f:
+                if ln.lower().startswith(("model name", "cpu part")):
+                    return ln.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    return "unknown"
+
+
+# ---------------------------------------------------------------- arms
+def run_dkv(args, dist):
+    import torch
+
+    import paper_2609_32663_gb300.dkv as dkv
+    from paper_2609_32663_gb300 import build
+    build.build_library()
+    dev = torch.device("cuda", dist.local)
+    torch.cuda.set_device(dev)
+    wl = I.WORKLOADS[args.workload]
+    steps, warmup = args.steps, max(args.warmup, 3)
+    if args.profile:
+        steps, warmup = min(steps, 2), min(warmup, 3)
+    reserve = steps + warmup + 64
+    env = setup(wl, dev, reserve)
+    comp = time_compaction(env, reps=3 if args.profile else 10)
+    info = env["info"]
+    NHl = wl.B * wl.Hkv
+    ln, *_ = dkv.dkv_plan_read(env["plan"])
+    rows_layer = [int(ln[l * NHl:(l + 1) * NHl].sum()) for l in range(wl.L)]
+
+    runner = DecodeRunner(wl, env["plan"], env["Kc"], env["Vc"], dev)
+    runner.capture()
+    clocks = Clocks(dist.local)
+    t_step, clk = time_graph(runner, steps, warmup, dist, clocks)
+    t_step = dist.max(t_step)
+    # Rows attended per step (the cache grows by one row per slab per step).
+    napp_mid = warmup + (steps - 1) / 2.0
+    rows_step = sum(rows_layer) + wl.L * NHl * (napp_mid + 1)
+    algo_step = step_bytes(wl, rows_step)
+
+    # Dominant kernel: the split-K partial pass, per launch (one layer).
+    n_inst = 4 if args.profile else 16
+    before = runner.n_app.clone()
+    t_part, n_launch = runner.timed_partials(n_inst)
+    napp_inst = float(before[0].item()) + (n_inst - 1) / 2.0
+    rows_launch = (sum(rows_layer) + wl.L * NHl * (napp_inst + 1)) / wl.L
+    part_bytes = rows_launch * 512 + wl.B * wl.H * 256 + 4 * wl.B * wl.Hkv * 256
+    peaks, src = measured_peaks()
+    peak = float(peaks["hbm_gbs"])
+    achieved = part_bytes / t_part / 1e9
+
+    res = {
+        "metric": METRIC, "value": round(t_step * 1e6, 2), "unit": UNIT, "n_gpus": dist.world,
+        "steps": steps, "warmup": warmup, "ms_per_step": round(t_step * 1e3, 4),
+        "higher_is_better": False, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "io_dtype": "bf16", "data": "synthetic",
+        "config": {"workload": wl.name, "layers": wl.L, "q_heads": wl.H, "kv_heads": wl.Hkv, "head_dim": wl.head_dim,
+                   "batch": wl.B, "ctx_len": [int(x) for x in env["Tc"]][:16], "bins": wl.D, "bin_width": wl.W,
+                   "sink": wl.sink, "recent": wl.recent,
+                   "physical_retention": round(info.kept_rows / (wl.L * wl.Hkv * float(env["Tc"].sum())), 4),
+                   "logical_retention": round(float(env["M"].mean()), 4),
+                   "parallelism": f"replicas x{dist.world}",
+                   "l2": "inputs larger than L2 (%.2f GB of K/V per step)" % (rows_step * 512 / 1e9),
+                   "graph": "one CUDA graph per step: %d layers x (partial + combine) + advance" % wl.L},
+        "tokens_per_s": round(wl.B * dist.world / t_step, 1),
+        "algorithmic_gb_per_step": round(algo_step / 1e9, 4),
+        "step_gbs": round(algo_step / t_step / 1e9, 1),
+        "step_frac_of_hbm": round(algo_step / t_step / 1e9 / peak, 4),
+        "roofline": {"bound": "hbm", "kernel": "decode_partial_kernel", "achieved": round(achieved, 1),
+                     "peak": peak, "unit": "GB/s", "frac": round(achieved / peak, 4), "peak_source": src,
+                     "frac_of_nominal_8000": round(achieved / 8000.0, 4),
+                     "bytes_per_launch": int(part_bytes), "avg_launch_us": round(t_part * 1e6, 2),
+                     "launches_timed": n_launch, "traffic": None},
+        "compaction": {"gbs": round(comp["gbs"], 1), "ms": round(comp["ms"], 3),
+                       "frac_of_hbm": round(comp["gbs"] / peak, 4), "kept_rows": info.kept_rows},
+        "map_ms": round(env["map_ms"], 2),
+        "gpu_launches": steps * (2 * wl.L + 1),
+        "clocks": clk,
+    }
+    del runner
+
+    if not args.no_dense and not args.profile:
+        dense = dkv.dkv_plan_dense(env["Tc"], env["shape"], T_stride=env["T_stride"])
+        dr = DecodeRunner(wl, dense, env["K"], env["V"], dev)
+        dr.capture()
+        t_dense, _ = time_graph(dr, steps, warmup, dist)
+        t_dense = dist.max(t_dense)
+        dense_rows = wl.L * float(env["Tc"].sum()) * wl.Hkv + wl.L * NHl * (napp_mid + 1)
+        res["dense_baseline"] = {"us_per_step": round(t_dense * 1e6, 2),
+                                 "gbs": round(step_bytes(wl, dense_rows) / t_dense / 1e9, 1),
+                                 "speedup_of_compacted": round(t_dense / t_step, 3),
+                                 "ideal_speedup": round(dense_rows / rows_step, 3)}
+        del dr
+        dense.close()
+
+    # End to end through the public API with host buffers (fresh plan state).
+    env2_plan = env["plan"]
+    t_e2e, bi, bo = run_e2e(wl, env2_plan, env["Kc"], env["Vc"], dev, max(8, min(steps, 32)), warmup)
+    t_e2e = dist.max(t_e2e)
+    res["e2e"] = {"value": round(t_e2e * 1e6, 2), "unit": UNIT, "h2d_bytes_per_step": int(bi),
+                  "d2h_bytes_per_step": int(bo), "steps": max(8, min(steps, 32)),
+                  "how": "CUDA graph of: H2D q/k_new/v_new from pinned host, L x dkv_decode_attn, dkv_advance, "
+                         "D2H of all layers' outputs"}
+
+    if dist.rank == 0 and dist.world == 1 and not args.no_cpu and not args.profile:
+        layers = max(1, min(args.cpu_layers, wl.L))
+        t_cpu, rows = cpu_oracle_step(wl, env, layers, dev)
+        res["cpu_baseline"] = {"value": round(t_cpu * 1e6, 1), "unit": UNIT, "cores": 1, "kind": "oracle",
+                               "sample": f"fp64 scalar oracle, {layers} of {wl.L} layers of one decode step "
+                                         f"({rows} rows x G={wl.G} heads), scaled x{wl.L / layers:g} to a step",
+                               "cpu": cpu_model(), "nproc": os.cpu_count()}
+    st = dkv.dkv_plan_status(env["plan"])
+    res["device_status_word"] = st
+    env["plan"].close()
+    return res
+
+
+def run_reference(args, dist):
+    """The oracle as it stands, timed on the host cores, per decode step of the
+    same workload (bounded sample of layers per step, scaled to a full step)."""
+    import oracle as O
+    wl = I.WORKLOADS[args.workload]
+    geo = O.Geometry(L=wl.L, H=wl.H, Hkv=wl.Hkv, D=wl.D, sink=wl.sink, recent=wl.recent, bin_width=wl.W)
+    M = I.make_pattern(wl)
+    Tc = I.context_lengths(wl)
+    layers = 1
+    # Map + pack of one layer's slabs (sample), then decode steps over that layer.
+    sub = O.Geometry(L=layers, H=wl.H, Hkv=wl.Hkv, D=wl.D, sink=wl.sink, recent=wl.recent, bin_width=wl.W)
+    m = O.map_pattern(M[:layers], Tc, sub, reserve=args.steps + args.warmup + 1)
+    rng = np.random.default_rng(wl.seed)
+    NHl = wl.B * wl.Hkv
+    Kc = rng.integers(0x3c00, 0x3f00, size=(m.total_rows, wl.head_dim), dtype=np.uint16)
+    Vc = rng.integers(0x3c00, 0x3f00, size=(m.total_rows, wl.head_dim), dtype=np.uint16)
+    q = rng.integers(0x3c00, 0x3f00, size=(wl.B, wl.H, wl.head_dim), dtype=np.uint16)
+    steps, warmup = max(1, min(args.steps, 3)), min(args.warmup, 1)
+    times = []
+    for i in range(warmup + steps):
+        t0 = time.perf_counter()
+        O.decode(m, 0, wl.B, wl.H, wl.Hkv, q, Kc, Vc)
+        if i >= warmup:
+            times.append((time.perf_counter() - t0) * wl.L / layers)
+    t = statistics.mean(times)
+    _ = geo, NHl
+    return {"impl": "reference", "metric": METRIC, "value": round(t * 1e6, 1), "unit": UNIT, "n_gpus": dist.world,
+            "steps": steps, "warmup": warmup, "ms_per_step": round(t * 1e3, 3), "higher_is_better": False,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": wl.name, "layers": wl.L, "q_heads": wl.H, "kv_heads": wl.Hkv, "batch": wl.B,
+                       "ctx_len": [int(x) for x in Tc][:16]},
+            "cpu_baseline": {"value": round(t * 1e6, 1), "unit": UNIT, "kind": "oracle", "cores": 1,
+                             "sample": f"{layers} of {wl.L} layers per step (all its KV heads), scaled to a step",
+                             "cpu": cpu_model(), "nproc": os.cpu_count()},
+            "e2e": {"value": round(t * 1e6, 1), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    args = parse()
+    dist = Dist(args.gpus)
+    try:
+        if args.impl == "reference":
+            if dist.rank != 0:
+                return
+            res = run_reference(args, dist)
+        else:
+            res = run_dkv(args, dist)
+        if dist.rank == 0:
+            print(json.dumps(res), flush=True)
+    finally:
+        dist.close()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,87 @@
+// Internal declarations shared by the translation units of libdkv.so.
+// Nothing here is part of the public ABI (include/dkv.h is).
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace dkv {
+
+constexpr int kHeadDim = 128;   // elements per row
+constexpr int kRowBytes = 256;  // bytes per bf16 row
+
+// ---------------------------------------------------------------- pattern map
+struct MapArgs {
+    const uint8_t* M;       // [L][H][D]
+    uint8_t* U;             // [L][Hkv][D], union over each GQA group
+    const int32_t* Tc;      // [B]
+    int32_t* chunk_cnt;     // [NH][nchunks], kept count of each position chunk
+    int32_t* len;           // [NH]
+    int64_t* off;           // [NH+1]
+    int64_t* ioff;          // [NH+1]
+    int32_t* idx;           // [kept]
+    int L, H, Hkv, D, B, sink, recent, bin_width, reserve;
+    int nchunks;            // position chunks per slab
+    int NH;                 // L*B*Hkv
+};
+constexpr int kMapChunk = 8192;  // positions per CTA in the count/write passes
+
+// Union, per-chunk counts and the offset scan; then, once idx is allocated, the writes.
+cudaError_t launch_map(const MapArgs& a, cudaStream_t st);
+cudaError_t launch_map_write(const MapArgs& a, cudaStream_t st);
+
+// ---------------------------------------------------------------- compaction
+struct CompactArgs {
+    const int32_t* len;
+    const int64_t* off;
+    const int64_t* ioff;
+    const int32_t* idx;
+    const uint16_t* K;
+    const uint16_t* V;
+    uint16_t* Kc;
+    uint16_t* Vc;
+    int64_t T_stride;
+    int64_t kept;
+    int NH;
+};
+cudaError_t launch_compact(const CompactArgs& a, cudaStream_t st);
+
+// ---------------------------------------------------------------- decode
+struct DecodeArgs {
+    const uint16_t* q;      // [B][H][128] bf16 bits
+    const uint16_t* k_new;  // [B][Hkv][128] or null
+    const uint16_t* v_new;
+    const int32_t* n_app;   // [B] or null
+    uint16_t* Kc;
+    uint16_t* Vc;
+    const int32_t* len;     // layer slice [NHl]
+    const int64_t* off;     // layer slice [NHl]
+    const int64_t* ioff;    // layer slice [NHl+1] (absolute; the layer prefix is ioff[h]-ioff[0])
+    float* work_o;          // [slots][G][128]
+    float* work_ml;         // [slots][G][2]
+    float* out;             // [B][H][128]
+    int32_t* status;
+    int B, H, Hkv, G;
+    int reserve;
+    int append;             // 1 when k_new/v_new are given
+    float qscale;           // softmax scale * log2(e)
+    int nctas;              // CTAs of the split-K grid (the partition's P)
+};
+
+// Slots of split-K partials a decode call can write: nctas + heads per layer.
+inline int64_t decode_slots(int nctas, int heads_per_layer) {
+    return (int64_t)nctas + heads_per_layer;
+}
+
+struct DecodeConfig {
+    int nctas;        // grid of the partial kernel
+    int smem_bytes;   // dynamic shared memory of the partial kernel
+};
+// Grid and shared memory of the partial kernel for group size G on this device.
+cudaError_t decode_config(int G, int B, DecodeConfig* cfg);
+// Split-K partials of one layer into the workspace, then the per-(b, q-head) merge.
+cudaError_t launch_decode_partial(const DecodeArgs& a, const DecodeConfig& cfg, cudaStream_t st);
+cudaError_t launch_decode_combine(const DecodeArgs& a, cudaStream_t st);
+cudaError_t launch_advance(int32_t* n_app, int B, int reserve, int32_t* status, cudaStream_t st);
+
+}  // namespace dkv

@@ -1,0 +1,246 @@
+"""Thin Python binding of the C ABI in include/dkv.h (libdkv.so).
+
+Argument marshalling only: each function takes torch tensors (device buffers)
+or numpy arrays (host inputs), passes raw pointers, sizes and the current CUDA
+stream to the function of the same name in libdkv.so, and raises DkvError on a
+non-zero status. Every step of the path runs in the library's CUDA kernels;
+there is no Python or CPU fallback, and importing the functions fails loudly
+when libdkv.so has not been built.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+
+import numpy as np
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libdkv.so")
+
+DKV_OK, DKV_ERR_INVALID_ARG, DKV_ERR_CUDA, DKV_ERR_OOM, DKV_ERR_RANGE, DKV_ERR_TIMEOUT = range(6)
+DKV_DEV_APPEND_OVERFLOW = 0x1
+DKV_DEV_TMA_TIMEOUT = 0x2
+
+# Every entry point include/dkv.h declares.
+EXPORTS = ("dkv_last_error", "dkv_map_pattern", "dkv_plan_dense", "dkv_plan_query", "dkv_plan_read",
+           "dkv_compact", "dkv_decode_attn", "dkv_decode_partial", "dkv_decode_combine", "dkv_advance",
+           "dkv_plan_status", "dkv_free")
+
+
+class DkvError(RuntimeError):
+    def __init__(self, status, func, msg):
+        super().__init__(f"{func} failed with status {status}: {msg}")
+        self.status = status
+
+
+class dkv_shape(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in
+                ("L", "H", "H_kv", "D", "head_dim", "sink", "recent", "bin_width")]
+
+
+@dataclass(frozen=True)
+class Shape:
+    """Model and pattern geometry (dkv_shape)."""
+    L: int
+    H: int
+    H_kv: int
+    D: int
+    head_dim: int = 128
+    sink: int = 128
+    recent: int = 1024
+    bin_width: int = 128
+
+    def c(self):
+        return dkv_shape(self.L, self.H, self.H_kv, self.D, self.head_dim, self.sink, self.recent,
+                         self.bin_width)
+
+    @property
+    def G(self):
+        return self.H // self.H_kv
+
+
+_lib = None
+
+
+def lib(path: str | None = None):
+    """Load libdkv.so (once) and declare its signatures."""
+    global _lib
+    if _lib is not None and path is None:
+        return _lib
+    p = path or LIB_PATH
+    if not os.path.exists(p):
+        raise RuntimeError(f"{p} is missing: build it with paper_2609_32663_gb300.build.build_library() "
+                           "(or __graft_entry__.build()); there is no fallback path")
+    L = ctypes.CDLL(p)
+    V, I32, I64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
+    PP = ctypes.POINTER(ctypes.c_void_p)
+    L.dkv_last_error.restype = ctypes.c_char_p
+    L.dkv_last_error.argtypes = []
+    L.dkv_map_pattern.restype = ctypes.c_int
+    L.dkv_map_pattern.argtypes = [V, V, I32, ctypes.POINTER(dkv_shape), I32, V, PP]
+    L.dkv_plan_dense.restype = ctypes.c_int
+    L.dkv_plan_dense.argtypes = [V, I32, ctypes.POINTER(dkv_shape), I64, V, PP]
+    L.dkv_plan_query.restype = ctypes.c_int
+    L.dkv_plan_query.argtypes = [V, ctypes.POINTER(I64), ctypes.POINTER(I64), PP, PP, PP, PP]
+    L.dkv_plan_read.restype = ctypes.c_int
+    L.dkv_plan_read.argtypes = [V, V, V, V, V, V]
+    L.dkv_compact.restype = ctypes.c_int
+    L.dkv_compact.argtypes = [V, V, V, I64, V, V, V]
+    L.dkv_decode_attn.restype = ctypes.c_int
+    L.dkv_decode_attn.argtypes = [V, I32, V, V, V, V, V, V, ctypes.c_float, V, V]
+    L.dkv_decode_partial.restype = ctypes.c_int
+    L.dkv_decode_partial.argtypes = [V, I32, V, V, V, V, V, V, ctypes.c_float, V]
+    L.dkv_decode_combine.restype = ctypes.c_int
+    L.dkv_decode_combine.argtypes = [V, I32, V, I32, V, V]
+    L.dkv_advance.restype = ctypes.c_int
+    L.dkv_advance.argtypes = [V, V, V]
+    L.dkv_plan_status.restype = ctypes.c_int
+    L.dkv_plan_status.argtypes = [V, ctypes.POINTER(I32), I32, V]
+    L.dkv_free.restype = None
+    L.dkv_free.argtypes = [V]
+    if path is None:
+        _lib = L
+    return L
+
+
+def _check(status, func):
+    if status != DKV_OK:
+        raise DkvError(status, func, lib().dkv_last_error().decode(errors="replace"))
+
+
+def _ptr(t):
+    """Device (torch) or host (numpy) buffer -> address; None -> NULL."""
+    if t is None:
+        return None
+    if isinstance(t, np.ndarray):
+        return t.ctypes.data
+    return t.data_ptr()
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        if not torch.cuda.is_available():
+            return None
+        return torch.cuda.current_stream().cuda_stream
+    return stream if isinstance(stream, int) else stream.cuda_stream
+
+
+class Plan:
+    """Owner of a dkv_plan*; dkv_free runs on close() or garbage collection."""
+
+    def __init__(self, handle, shape: Shape, B: int, dense: bool):
+        self.handle = handle
+        self.shape = shape
+        self.B = B
+        self.dense = dense
+
+    def close(self):
+        if self.handle:
+            lib().dkv_free(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    @property
+    def _as_parameter_(self):
+        if not self.handle:
+            raise ValueError("plan already freed")
+        return ctypes.c_void_p(self.handle)
+
+
+def dkv_map_pattern(M, ctx_len, shape: Shape, reserve_rows: int = 0, stream=None) -> Plan:
+    M = np.ascontiguousarray(M, dtype=np.uint8)
+    ctx = np.ascontiguousarray(ctx_len, dtype=np.int32)
+    out = ctypes.c_void_p()
+    sh = shape.c()
+    _check(lib().dkv_map_pattern(_ptr(M), _ptr(ctx), len(ctx), ctypes.byref(sh), int(reserve_rows),
+                                 _stream(stream), ctypes.byref(out)), "dkv_map_pattern")
+    return Plan(out.value, shape, len(ctx), False)
+
+
+def dkv_plan_dense(ctx_len, shape: Shape, T_stride: int, stream=None) -> Plan:
+    ctx = np.ascontiguousarray(ctx_len, dtype=np.int32)
+    out = ctypes.c_void_p()
+    sh = shape.c()
+    _check(lib().dkv_plan_dense(_ptr(ctx), len(ctx), ctypes.byref(sh), int(T_stride), _stream(stream),
+                                ctypes.byref(out)), "dkv_plan_dense")
+    return Plan(out.value, shape, len(ctx), True)
+
+
+@dataclass
+class PlanInfo:
+    total_rows: int
+    kept_rows: int
+    d_len: int
+    d_off: int
+    d_ioff: int | None
+    d_idx: int | None
+
+
+def dkv_plan_query(plan: Plan) -> PlanInfo:
+    tr, kr = ctypes.c_int64(), ctypes.c_int64()
+    pl, po, pi, px = (ctypes.c_void_p() for _ in range(4))
+    _check(lib().dkv_plan_query(plan, ctypes.byref(tr), ctypes.byref(kr), ctypes.byref(pl),
+                                ctypes.byref(po), ctypes.byref(pi), ctypes.byref(px)), "dkv_plan_query")
+    return PlanInfo(tr.value, kr.value, pl.value, po.value, pi.value, px.value)
+
+
+def dkv_compact(plan: Plan, K, V, Kc, Vc, T_stride: int | None = None, stream=None):
+    if T_stride is None:
+        T_stride = K.shape[-2]
+    _check(lib().dkv_compact(plan, _ptr(K), _ptr(V), int(T_stride), _ptr(Kc), _ptr(Vc), _stream(stream)),
+           "dkv_compact")
+
+
+def dkv_decode_attn(plan: Plan, layer: int, q, k_new, v_new, n_appended, Kc, Vc, out, scale: float = 0.0,
+                    stream=None):
+    _check(lib().dkv_decode_attn(plan, int(layer), _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(n_appended),
+                                 _ptr(Kc), _ptr(Vc), ctypes.c_float(scale), _ptr(out), _stream(stream)),
+           "dkv_decode_attn")
+
+
+def dkv_decode_partial(plan: Plan, layer: int, q, k_new, v_new, n_appended, Kc, Vc, scale: float = 0.0,
+                       stream=None):
+    _check(lib().dkv_decode_partial(plan, int(layer), _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(n_appended),
+                                    _ptr(Kc), _ptr(Vc), ctypes.c_float(scale), _stream(stream)),
+           "dkv_decode_partial")
+
+
+def dkv_decode_combine(plan: Plan, layer: int, n_appended, with_new_token: bool, out, stream=None):
+    _check(lib().dkv_decode_combine(plan, int(layer), _ptr(n_appended), int(bool(with_new_token)), _ptr(out),
+                                    _stream(stream)), "dkv_decode_combine")
+
+
+def dkv_advance(plan: Plan, n_appended, stream=None):
+    _check(lib().dkv_advance(plan, _ptr(n_appended), _stream(stream)), "dkv_advance")
+
+
+def dkv_plan_status(plan: Plan, clear: bool = False, stream=None) -> int:
+    w = ctypes.c_int32()
+    _check(lib().dkv_plan_status(plan, ctypes.byref(w), int(bool(clear)), _stream(stream)), "dkv_plan_status")
+    return w.value
+
+
+def dkv_free(plan: Plan):
+    plan.close()
+
+
+def dkv_plan_read(plan: Plan, stream=None):
+    """Host copies (numpy) of the plan's len, off, ioff and idx arrays."""
+    info = dkv_plan_query(plan)
+    NH = plan.shape.L * plan.B * plan.shape.H_kv
+    ln = np.zeros(NH, np.int32)
+    off = np.zeros(NH + 1, np.int64)
+    ioff = np.zeros(NH + 1, np.int64)
+    idx = np.zeros(max(info.kept_rows, 1), np.int32)
+    _check(lib().dkv_plan_read(plan, _ptr(ln), _ptr(off), _ptr(ioff), _ptr(idx), _stream(stream)),
+           "dkv_plan_read")
+    if plan.dense:
+        return ln, off, None, None
+    return ln, off, ioff, idx[: info.kept_rows]

@@ -1,0 +1,116 @@
+"""The C ABI library builds, loads and exports every declared entry point, and its
+host-side argument checks answer without a GPU (no kernel is launched here)."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def dkvmod():
+    from paper_2609_32663_gb300 import build
+    build.build_library()
+    import paper_2609_32663_gb300.dkv as dkv
+    return dkv
+
+
+def declared_functions():
+    src = open(os.path.join(ROOT, "include", "dkv.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(dkv_\w+)\s*\(", src)))
+
+
+def test_header_declares_the_binding_exports(dkvmod):
+    assert declared_functions() == sorted(dkvmod.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol(dkvmod):
+    lib = ctypes.CDLL(dkvmod.LIB_PATH)
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_library_is_built_for_sm_103a_only():
+    from paper_2609_32663_gb300 import build
+    assert build.ARCH == ["-gencode", "arch=compute_103a,code=sm_103a"]
+
+
+def _shape(dkv, **kw):
+    base = dict(L=2, H=8, H_kv=2, D=4, sink=2, recent=3, bin_width=5)
+    base.update(kw)
+    return dkv.Shape(**base)
+
+
+@pytest.mark.parametrize("kw,ctx,status", [
+    (dict(H=6, H_kv=4), [10], "INVALID_ARG"),           # H % H_kv != 0
+    (dict(head_dim=64), [10], "INVALID_ARG"),            # only 128
+    (dict(H=18, H_kv=2), [10], "INVALID_ARG"),           # group size 9 > 8
+    (dict(bin_width=0), [10], "INVALID_ARG"),
+    (dict(), [-1], "INVALID_ARG"),                       # negative length
+    (dict(), [2 + 3 + 4 * 5 + 1], "RANGE"),              # needs a 5th bin
+])
+def test_map_pattern_rejects_bad_arguments(dkvmod, kw, ctx, status):
+    dkv = dkvmod
+    sh = _shape(dkv, **kw)
+    M = np.zeros((sh.L, sh.H, sh.D), np.uint8)
+    with pytest.raises(dkv.DkvError) as e:
+        dkv.dkv_map_pattern(M, ctx, sh, stream=0)
+    assert e.value.status == getattr(dkv, "DKV_ERR_" + status)
+    assert dkv.lib().dkv_last_error()
+
+
+def test_map_pattern_rejects_non_binary_pattern(dkvmod):
+    dkv = dkvmod
+    sh = _shape(dkv)
+    M = np.zeros((sh.L, sh.H, sh.D), np.uint8)
+    M[1, 3, 2] = 7
+    with pytest.raises(dkv.DkvError) as e:
+        dkv.dkv_map_pattern(M, [10], sh, stream=0)
+    assert e.value.status == dkv.DKV_ERR_INVALID_ARG
+    assert b"M[" in dkv.lib().dkv_last_error()
+
+
+def test_null_arguments(dkvmod):
+    dkv = dkvmod
+    L = dkv.lib()
+    out = ctypes.c_void_p(123)
+    sh = _shape(dkv).c()
+    assert L.dkv_map_pattern(None, None, 1, ctypes.byref(sh), 0, None, ctypes.byref(out)) == dkv.DKV_ERR_INVALID_ARG
+    assert out.value is None
+    assert L.dkv_map_pattern(None, None, 1, ctypes.byref(sh), 0, None, None) == dkv.DKV_ERR_INVALID_ARG
+    assert L.dkv_compact(None, None, None, 1, None, None, None) == dkv.DKV_ERR_INVALID_ARG
+    assert L.dkv_decode_attn(None, 0, None, None, None, None, None, None, ctypes.c_float(0), None, None) == \
+        dkv.DKV_ERR_INVALID_ARG
+    assert L.dkv_advance(None, None, None) == dkv.DKV_ERR_INVALID_ARG
+    assert L.dkv_plan_query(None, None, None, None, None, None, None) == dkv.DKV_ERR_INVALID_ARG
+    L.dkv_free(None)  # NULL-safe
+
+
+def test_injected_allocation_failure_reports_oom(dkvmod, monkeypatch):
+    """Host-side fault injection: the first device allocation fails before any
+    CUDA call, and the error surfaces as DKV_ERR_OOM with a message."""
+    dkv = dkvmod
+    monkeypatch.setenv("DKV_FAULT", "alloc")
+    sh = _shape(dkv)
+    M = np.ones((sh.L, sh.H, sh.D), np.uint8)
+    with pytest.raises(dkv.DkvError) as e:
+        dkv.dkv_map_pattern(M, [12, 20], sh, stream=0)
+    assert e.value.status == dkv.DKV_ERR_OOM
+    assert b"injected" in dkv.lib().dkv_last_error()
+
+
+def test_dense_plan_rejects_short_stride(dkvmod):
+    dkv = dkvmod
+    with pytest.raises(dkv.DkvError) as e:
+        dkv.dkv_plan_dense([100, 300], _shape(dkv), T_stride=200, stream=0)
+    assert e.value.status == dkv.DKV_ERR_INVALID_ARG
+
+
+def test_binding_fails_loudly_without_library(tmp_path):
+    import paper_2609_32663_gb300.dkv as dkv
+    with pytest.raises(RuntimeError, match="missing"):
+        dkv.lib(str(tmp_path / "libdkv.so"))
