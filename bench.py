@@ -99,9 +99,13 @@ class Clocks:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
-                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+                 "-lms", "20"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.t = threading.Thread(target=self._read, daemon=True)
             self.t.start()
+            t0 = time.time()
+            while not self.lines and time.time() - t0 < 3.0 and self.proc.poll() is None:
+                time.sleep(0.01)  # the sampler is running before the timed region starts
+            self.lines.clear()
         except (OSError, FileNotFoundError):
             self.proc = None
 
@@ -268,7 +272,6 @@ def time_graph(runner, steps, warmup, dist, clocks=None):
     torch.cuda.synchronize()
     if clocks:
         clocks.start()
-        time.sleep(0.3)
     st = torch.cuda.current_stream()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(st)
