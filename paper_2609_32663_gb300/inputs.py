@@ -66,6 +66,11 @@ WORKLOADS = {
     "llama8b-128k": Workload("llama8b-128k", L=32, H=32, Hkv=8, T=131072, B=1, D=128,
                              W=_w(131072, 128), pattern="profile", rate=0.346,
                              physical_target=0.346, outlier_frac=0.01, seed=3),
+    # Same head shape, pattern recipe and per-layer sizes as llama8b-128k, 4 layers only:
+    # a small case (about 3 GB on the device) for detailed profiles of the same kernels.
+    "llama8b-128k-l4": Workload("llama8b-128k-l4", L=4, H=32, Hkv=8, T=131072, B=1, D=128,
+                                W=_w(131072, 128), pattern="profile", rate=0.346,
+                                physical_target=0.346, outlier_frac=0.01, seed=3),
     "llama8b-b16-ragged": Workload("llama8b-b16-ragged", L=32, H=32, Hkv=8, T=65536, B=16, D=64,
                                    W=_w(65536, 64), pattern="profile", rate=0.25,
                                    ragged=(8192, 65536), seed=4),
