@@ -209,6 +209,33 @@ dkv_status dkv_advance(const dkv_plan* plan, int32_t* n_appended, cudaStream_t s
  */
 dkv_status dkv_plan_status(const dkv_plan* plan, int32_t* word, int32_t clear, cudaStream_t stream);
 
+/*
+ * dkv_decode_attn without any device allocation. The paper has no counterpart:
+ * this is for callers that must not allocate device memory -- code hosted by a
+ * serving engine or plugin framework that owns the whole device pool and
+ * forbids cudaMalloc/cudaFree (both synchronise the device and fragment the
+ * pool). Such callers cannot build a dkv_plan, so they pass the plan's metadata
+ * themselves, laid out as dkv_plan_query describes:
+ *   d_len  int32 [L*B*H_kv], d_off and d_ioff int64 [L*B*H_kv + 1] (device),
+ * with reserve_rows the free rows after every slab. All other arguments are
+ * those of dkv_decode_attn. status is a device int32 that receives the
+ * DKV_DEV_* bits, or NULL to discard them.
+ *
+ * The split-K partials live in a fixed 8 MiB array inside the library image,
+ * held on every GPU that loads the library until the process exits; a call
+ * whose partials ((SM-count CTAs + B*H_kv) x G x 130 floats) do not fit gets
+ * DKV_ERR_INVALID_ARG. The first call on each device looks up that array's
+ * device address (a one-time set-up per device); make that first call before
+ * any stream capture. Every call reuses the same array, so calls whose kernels
+ * overlap on the GPU (other streams, other threads) race with each other.
+ * Errors: DKV_ERR_INVALID_ARG, DKV_ERR_CUDA.
+ */
+dkv_status dkv_decode_attn_noalloc(const dkv_shape* s, int32_t B, int32_t layer, int32_t reserve_rows,
+                                   const int32_t* d_len, const int64_t* d_off, const int64_t* d_ioff,
+                                   const void* q, const void* k_new, const void* v_new,
+                                   const int32_t* n_appended, void* Kc, void* Vc, float scale,
+                                   float* out, int32_t* status, cudaStream_t stream);
+
 /* Release a plan (NULL-safe). Synchronises the device before freeing. */
 void dkv_free(dkv_plan* plan);
 

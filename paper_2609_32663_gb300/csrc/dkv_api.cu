@@ -137,6 +137,15 @@ dkv_status finish_plan(dkv_plan* p)
 
 }  // namespace
 
+namespace dkv {
+// Lets other translation units of the library report through dkv_last_error().
+dkv_status set_error(dkv_status st, const char* msg)
+{
+    snprintf(g_err, sizeof g_err, "%s", msg ? msg : "");
+    return st;
+}
+}  // namespace dkv
+
 extern "C" {
 
 const char* dkv_last_error(void) { return g_err; }

@@ -25,7 +25,7 @@ DKV_DEV_TMA_TIMEOUT = 0x2
 # Every entry point include/dkv.h declares.
 EXPORTS = ("dkv_last_error", "dkv_map_pattern", "dkv_plan_dense", "dkv_plan_query", "dkv_plan_read",
            "dkv_compact", "dkv_decode_attn", "dkv_decode_partial", "dkv_decode_combine", "dkv_advance",
-           "dkv_plan_status", "dkv_free")
+           "dkv_plan_status", "dkv_free", "dkv_decode_attn_noalloc")
 
 
 class DkvError(RuntimeError):
@@ -97,6 +97,9 @@ def lib(path: str | None = None):
     L.dkv_advance.argtypes = [V, V, V]
     L.dkv_plan_status.restype = ctypes.c_int
     L.dkv_plan_status.argtypes = [V, ctypes.POINTER(I32), I32, V]
+    L.dkv_decode_attn_noalloc.restype = ctypes.c_int
+    L.dkv_decode_attn_noalloc.argtypes = [ctypes.POINTER(dkv_shape), I32, I32, I32, V, V, V, V, V, V, V, V, V,
+                                          ctypes.c_float, V, V, V]
     L.dkv_free.restype = None
     L.dkv_free.argtypes = [V]
     if path is None:
@@ -229,6 +232,18 @@ def dkv_plan_status(plan: Plan, clear: bool = False, stream=None) -> int:
 
 def dkv_free(plan: Plan):
     plan.close()
+
+
+def dkv_decode_attn_noalloc(shape: Shape, B: int, layer: int, reserve_rows: int, d_len, d_off, d_ioff, q, k_new,
+                            v_new, n_appended, Kc, Vc, out, scale: float = 0.0, status=None, stream=None):
+    """Decode attention that allocates no device memory; d_len/d_off/d_ioff are
+    device addresses (ints) or tensors of the plan metadata."""
+    sh = shape.c()
+    addr = (lambda t: t if isinstance(t, int) or t is None else _ptr(t))
+    _check(lib().dkv_decode_attn_noalloc(ctypes.byref(sh), int(B), int(layer), int(reserve_rows), addr(d_len),
+                                         addr(d_off), addr(d_ioff), _ptr(q), _ptr(k_new), _ptr(v_new),
+                                         _ptr(n_appended), _ptr(Kc), _ptr(Vc), ctypes.c_float(scale), _ptr(out),
+                                         _ptr(status), _stream(stream)), "dkv_decode_attn_noalloc")
 
 
 def dkv_plan_read(plan: Plan, stream=None):
