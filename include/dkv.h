@@ -80,7 +80,7 @@ const char* dkv_last_error(void);
  *
  * M_host        host uint8 [L][H][D], entries 0 or 1. Copied; caller keeps it.
  * ctx_len_host  host int32 [B], context length Tc[b] >= 0 of each sequence.
- * B             number of sequences, 1 <= B <= 1024.
+ * B             number of sequences, 1 <= B <= 512.
  * s             geometry; head_dim must be 128.
  * reserve_rows  free rows after every slab for appended tokens (>= 0).
  * stream        stream for the copies and kernels.

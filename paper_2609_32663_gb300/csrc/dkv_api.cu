@@ -116,7 +116,7 @@ dkv_status check_shape(const dkv_shape* s, int32_t B)
     if (s->sink < 0 || s->recent < 0 || s->bin_width < 1)
         return fail(DKV_ERR_INVALID_ARG, "bad sink/recent/bin_width: %d/%d/%d", s->sink, s->recent,
                     s->bin_width);
-    if (B < 1 || B > 1024) return fail(DKV_ERR_INVALID_ARG, "B=%d out of [1, 1024]", B);
+    if (B < 1 || B > 512) return fail(DKV_ERR_INVALID_ARG, "B=%d out of [1, 512]", B);
     return DKV_OK;
 }
 

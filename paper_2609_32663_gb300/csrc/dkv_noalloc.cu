@@ -79,7 +79,7 @@ extern "C" dkv_status dkv_decode_attn_noalloc(const dkv_shape* s, int32_t B, int
     if (s->L < 1 || s->H < 1 || s->H_kv < 1 || s->H % s->H_kv != 0 || s->H / s->H_kv > 8)
         return bad(DKV_ERR_INVALID_ARG, "bad head geometry H=%d H_kv=%d", s->H, s->H_kv);
     if (s->head_dim != dkv::kHeadDim) return bad(DKV_ERR_INVALID_ARG, "head_dim=%d: only 128", s->head_dim);
-    if (B < 1 || B > 1024) return bad(DKV_ERR_INVALID_ARG, "B=%d out of [1, 1024]", B);
+    if (B < 1 || B > 512) return bad(DKV_ERR_INVALID_ARG, "B=%d out of [1, 512]", B);
     if (layer < 0 || layer >= s->L) return bad(DKV_ERR_INVALID_ARG, "layer=%d out of [0, %d)", layer, s->L);
     if (reserve_rows < 0) return bad(DKV_ERR_INVALID_ARG, "reserve_rows=%d < 0", reserve_rows);
     if (!d_len || !d_off || !d_ioff || !q || !Kc || !Vc || !out)

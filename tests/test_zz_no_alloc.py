@@ -105,11 +105,11 @@ def test_noalloc_allocates_nothing(case):
 
 def test_noalloc_rejects_workspace_beyond_the_static_array(case):
     c = case
-    big = dkv.Shape(L=1, H=64, H_kv=8, D=1)  # 1024 sequences x 8 KV heads x G=8 partials > 8 MiB
+    big = dkv.Shape(L=1, H=64, H_kv=8, D=1)  # 512 sequences x 8 KV heads x G=8 partials > 8 MiB
     d_len, d_off, d_ioff = metadata(c)
-    out = torch.empty((1024, 64, 128), dtype=torch.float32, device=c.dev)
-    q = torch.zeros((1024, 64, 128), dtype=torch.bfloat16, device=c.dev)
+    out = torch.empty((512, 64, 128), dtype=torch.float32, device=c.dev)
+    q = torch.zeros((512, 64, 128), dtype=torch.bfloat16, device=c.dev)
     with pytest.raises(dkv.DkvError) as e:
-        dkv.dkv_decode_attn_noalloc(big, 1024, 0, 0, d_len, d_off, d_ioff, q, None, None, None, c.Kc, c.Vc, out)
+        dkv.dkv_decode_attn_noalloc(big, 512, 0, 0, d_len, d_off, d_ioff, q, None, None, None, c.Kc, c.Vc, out)
     assert e.value.status == dkv.DKV_ERR_INVALID_ARG
     assert b"static scratch" in dkv.lib().dkv_last_error()
