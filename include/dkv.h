@@ -171,6 +171,12 @@ dkv_status dkv_compact(const dkv_plan* plan, const void* K, const void* V, int64
  * The plan holds the split-K workspace, so calls with the same plan must be
  * ordered (same stream, or synchronised). An append past the reserve is skipped
  * and sets DKV_DEV_APPEND_OVERFLOW.
+ * The kernels use programmatic dependent launch: they may start while the
+ * previous kernel in the stream is still running, and read q, k_new, v_new only
+ * after it has completed. n_appended and the packed cache rows of earlier steps
+ * are read before that point, so they must not be written by the kernel that
+ * immediately precedes this call if that kernel signals early completion
+ * (griddepcontrol.launch_dependents); an ordinary kernel never does.
  * Errors: DKV_ERR_INVALID_ARG (NULL/unaligned pointer, layer out of range,
  * only one of k_new/v_new), DKV_ERR_CUDA.
  */
@@ -223,7 +229,8 @@ dkv_status dkv_plan_status(const dkv_plan* plan, int32_t* word, int32_t clear, c
  *
  * The split-K partials live in a fixed 8 MiB array inside the library image,
  * held on every GPU that loads the library until the process exits; a call
- * whose partials ((SM-count CTAs + B*H_kv) x G x 130 floats) do not fit gets
+ * whose split-K records ((17 x SM count + B*H_kv) x G x 130 floats for G <= 4,
+ * (9 x SM count + B*H_kv) x G x 130 for G > 4) do not fit gets
  * DKV_ERR_INVALID_ARG. The first call on each device looks up that array's
  * device address (a one-time set-up per device); make that first call before
  * any stream capture. Every call reuses the same array, so calls whose kernels

@@ -29,6 +29,7 @@ struct dkv_plan {
     int32_t* d_idx = nullptr;   // [kept]
     int32_t* d_status = nullptr;
     float* d_work = nullptr;    // split-K partials
+    int32_t* d_slab_count = nullptr;  // [B*H_kv] arrival counters of the fused combine
     dkv::DecodeConfig cfg{};
     int64_t slots = 0;
 };
@@ -99,6 +100,7 @@ void release(dkv_plan* p)
     cudaFree(p->d_idx);
     cudaFree(p->d_status);
     cudaFree(p->d_work);
+    cudaFree(p->d_slab_count);
     delete p;
 }
 
@@ -126,12 +128,17 @@ dkv_status finish_plan(dkv_plan* p)
     cudaGetDevice(&p->device);
     cudaError_t e = dkv::decode_config(p->G, p->B, &p->cfg);
     if (e != cudaSuccess) return cuda_fail(e, "decode_config");
-    p->slots = dkv::decode_slots(p->cfg.nctas, p->B * p->s.H_kv);
-    dkv_status st = dalloc(&p->d_work, (size_t)p->slots * p->G * (dkv::kHeadDim + 2), "split-K workspace");
+    p->slots = (int64_t)p->cfg.nctas + p->B * p->s.H_kv;
+    dkv_status st = dalloc(&p->d_work, (size_t)dkv::decode_workspace_floats(p->cfg, p->G, p->B * p->s.H_kv),
+                           "split-K workspace");
     if (st != DKV_OK) return st;
     st = dalloc(&p->d_status, 1, "status word");
     if (st != DKV_OK) return st;
     if ((e = cudaMemset(p->d_status, 0, sizeof(int32_t))) != cudaSuccess) return cuda_fail(e, "cudaMemset");
+    st = dalloc(&p->d_slab_count, (size_t)p->B * p->s.H_kv, "slab counters");
+    if (st != DKV_OK) return st;
+    if ((e = cudaMemset(p->d_slab_count, 0, sizeof(int32_t) * p->B * p->s.H_kv)) != cudaSuccess)
+        return cuda_fail(e, "cudaMemset");
     return DKV_OK;
 }
 
@@ -430,9 +437,13 @@ dkv_status decode_args(const dkv_plan* p, int32_t layer, const void* q, const vo
     a->len = p->d_len + (int64_t)layer * NHl;
     a->off = p->d_off + (int64_t)layer * NHl;
     a->ioff = p->d_ioff + (int64_t)layer * NHl;
+    const size_t nw = (size_t)p->cfg.nctas * p->cfg.nwarps;
     a->work_o = p->d_work;
-    a->work_ml = p->d_work + (size_t)p->slots * p->G * dkv::kHeadDim;
+    a->work_ml = a->work_o + (size_t)p->slots * p->G * dkv::kHeadDim;
+    a->warp_o = a->work_ml + (size_t)p->slots * p->G * 2;
+    a->warp_ml = a->warp_o + nw * p->G * dkv::kHeadDim;
     a->out = out;
+    a->slab_count = p->d_slab_count;
     a->status = p->d_status;
     a->B = p->B;
     a->H = p->s.H;
@@ -456,9 +467,7 @@ dkv_status dkv_decode_attn(const dkv_plan* p, int32_t layer, const void* q, cons
     dkv_status st = decode_args(p, layer, q, k_new, v_new, k_new != nullptr, n_appended, Kc, Vc, scale, out,
                                 true, true, &a);
     if (st != DKV_OK) return st;
-    if ((st = launched(dkv::launch_decode_partial(a, p->cfg, stream), "decode partial kernel")) != DKV_OK)
-        return st;
-    st = launched(dkv::launch_decode_combine(a, stream), "decode combine kernel");
+    st = launched(dkv::launch_decode_fused(a, p->cfg, stream), "decode kernel");
     return st == DKV_OK ? ok() : st;
 }
 

@@ -1,22 +1,25 @@
 // Decode-step attention over the packed cache (Sec. 3.4), split-K.
 //
 // Work split ("stream-K" over rows). For one layer, the rows of all slabs
-// h = b*Hkv + g are laid end to end: slab h owns global rows
-// [P(h), P(h+1)), n_h = len[h] + appended[b] (+1 for this step's token).
-// CTA c of P CTAs takes rows [A(c), A(c+1)), A(c) = floor(c*R/P), so every CTA
-// streams the same number of bytes whatever the slab lengths. It writes one
-// partial (m, l, o) per slab it touches into slot c + h; the slots are
-// distinct because CTA ranges and slabs are both in row order. The combine
-// kernel then merges, for each (b, q-head), the partials of the CTAs that
-// cover its slab.
+// h = b*Hkv + g are laid end to end: slab h owns layer rows [P(h), P(h+1)),
+// n_h = len[h] + appended[b] (+1 for this step's token). CTA c of P takes rows
+// [A(c), A(c+1)), A(c) = floor(c*R/P), so every CTA streams the same number of
+// bytes whatever the slab lengths; its warps split that range into equal
+// contiguous pieces and run independently (no barrier until the end). Each CTA
+// writes one partial (m, l, o) per slab it touches into slot c + h; the slots
+// are distinct because CTA ranges and slabs are both in row order. The combine
+// kernel merges, for each (b, q-head), the partials of the CTAs covering its slab.
 //
-// Inside a CTA, each warp owns a ring of NS stages and fetches its tiles of
-// TR rows (K and V, 256 bytes a row) with cp.async.bulk into shared memory,
-// completing on an mbarrier; tiles of a slab segment go round-robin to the
-// warps. A half-warp takes one row, a lane 8 dims: q.k is 8 FMAs per lane and
-// a 4-step xor-shuffle sum over the half, then an online softmax in base 2
-// (q is pre-scaled by scale*log2 e), and o += p v on the lane's 8 dims. At the
-// end of each slab segment the warps' states merge in shared memory.
+// A warp fetches its tiles of TR rows (K and V, 256 bytes a row) with
+// cp.async.bulk into its own ring of NS shared-memory stages, each completing
+// on an mbarrier. LPR lanes share a row (16 or 8 dims each): q.k partial sums
+// use packed f32x2 FMAs and are summed across the LPR lanes through a small
+// shared-memory transpose; the softmax is online in base 2 (scores scaled by
+// scale*log2 e) with one exp per (row, head); o += p v again in f32x2. A warp
+// keeps the state of its last slab in registers; the state of a slab it leaves
+// earlier goes to a per-warp record (first slab) or straight to the CTA's slot
+// (a slab wholly inside the warp's range). Warps do not wait for each other
+// until their ranges are done; then the CTA merges the states that share a slab.
 #include "dkv_internal.cuh"
 
 #include <math.h>
@@ -29,6 +32,7 @@ namespace {
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kMaxB = 512;
 constexpr int kWaitSpins = 1 << 22;  // bound on mbarrier polls (each poll may suspend)
+constexpr float kSlack = 8.f;        // lazy-rescale threshold of the online softmax (log2 units)
 
 // ------------------------------------------------------------ PTX helpers
 __device__ __forceinline__ uint32_t smem_u32(const void* p)
@@ -85,6 +89,18 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t
         : "memory");
 }
 
+// Programmatic dependent launch: let the next kernel in the stream start its
+// prologue, and wait for the previous kernel's results before reading them.
+__device__ __forceinline__ void pdl_launch_dependents()
+{
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+__device__ __forceinline__ void pdl_wait()
+{
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
 __device__ __forceinline__ void fence_proxy_async_smem()
 {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -93,7 +109,7 @@ __device__ __forceinline__ void fence_proxy_async_smem()
 // ------------------------------------------------------------ partition
 // Per-call sequence table in shared memory: NA[b] = rows already appended
 // (clamped to the reserve), NP[b] = exclusive prefix over b of the extra rows
-// e_b = NA[b] + (this call appends to b ? 1 : 0).
+// e_b = NA[b] + (this call appends to b ? 1 : 0). Layer rows fit in int32.
 struct SeqTable {
     int32_t* NA;  // [B]
     int32_t* NP;  // [B+1]
@@ -127,31 +143,34 @@ __device__ void build_seq_table(const DecodeArgs& a, SeqTable t, bool report)
     if (lane == 0) t.NP[a.B] = carry;
 }
 
-// First global row of slab h (h in [0, B*Hkv]) within this layer call.
-__device__ __forceinline__ int64_t slab_start(const DecodeArgs& a, const SeqTable& t, int h)
+// First layer row of slab h (h in [0, B*Hkv]) within this call.
+__device__ __forceinline__ int slab_start(const DecodeArgs& a, const SeqTable& t, int h)
 {
     const int b = h / a.Hkv, g = h - b * a.Hkv;
-    int64_t p = (a.ioff[h] - a.ioff[0]) + (int64_t)a.Hkv * t.NP[b];
-    if (g) p += (int64_t)g * (t.NP[b + 1] - t.NP[b]);
+    int p = (int)(a.ioff[h] - a.ioff[0]) + a.Hkv * t.NP[b];
+    if (g) p += g * (t.NP[b + 1] - t.NP[b]);
     return p;
 }
 
-__device__ __forceinline__ int64_t cta_start(int c, int64_t R, int P)
+__device__ __forceinline__ int part_start(int w, int R, int P)
 {
-    return ((int64_t)c * R) / P;
+    // floor(w R / P) without a 64-bit division: R = q P + r, so w R / P = w q + w r / P,
+    // and w r < P^2 fits 32 bits (P is a CTA count).
+    const unsigned q = (unsigned)R / (unsigned)P, r = (unsigned)R - q * (unsigned)P;
+    return (int)((unsigned)w * q + ((unsigned)w * r) / (unsigned)P);
 }
 
-// Largest c with cta_start(c) <= x, for 0 <= x < R.
-__device__ __forceinline__ int cta_of(int64_t x, int64_t R, int P)
+// Largest part w with part_start(w) <= x, for 0 <= x < R.
+__device__ __forceinline__ int part_of(int x, int R, int P)
 {
-    int c = (int)((x * P) / R);
-    while (c + 1 < P && cta_start(c + 1, R, P) <= x) ++c;
-    while (c > 0 && cta_start(c, R, P) > x) --c;
-    return c;
+    int w = (int)(((int64_t)x * P) / R);
+    while (w + 1 < P && part_start(w + 1, R, P) <= x) ++w;
+    while (w > 0 && part_start(w, R, P) > x) --w;
+    return w;
 }
 
 // Last slab h in [0, NHl) with slab_start(h) <= x.
-__device__ int slab_containing(const DecodeArgs& a, const SeqTable& t, int NHl, int64_t x)
+__device__ int slab_containing(const DecodeArgs& a, const SeqTable& t, int NHl, int x)
 {
     int lo = 0, hi = NHl - 1;
     while (lo < hi) {
@@ -214,10 +233,19 @@ __device__ __forceinline__ uint64_t bf2_to_f2(uint32_t w)
     return pk(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
 }
 
+__device__ __forceinline__ void bf8_to_f2x4(const uint4& w, uint64_t* out)
+{
+    out[0] = bf2_to_f2(w.x);
+    out[1] = bf2_to_f2(w.y);
+    out[2] = bf2_to_f2(w.z);
+    out[3] = bf2_to_f2(w.w);
+}
+
 // Compile-time geometry of the partial kernel.
-//   LPR lanes share one row (each owns DPL = 128/LPR dims, i.e. NCH 16-byte
-//   chunks c = s + LPR*i of the row); a warp step covers RPS = 32/LPR rows; a
-//   tile of TR rows takes STEPS steps. Scores: TR*G per tile, NSUM per lane.
+//   LPR lanes share one row; a lane owns DPL = 128/LPR dims, i.e. NCH 16-byte
+//   chunks c = sl + LPR*i of the row; a warp step covers RPS = 32/LPR rows; a
+//   tile of TR rows takes STEPS steps. A tile has TR*G scores, NSUM per lane:
+//   slot u of lane l is (row l % TR, head l / TR + u * 32/TR).
 template <int G_, int LPR_, int TR_, int NS_, int NW_>
 struct PK {
     static constexpr int G = G_, LPR = LPR_, TR = TR_, NS = NS_, NW = NW_;
@@ -225,437 +253,656 @@ struct PK {
     static constexpr int DPL = kHeadDim / LPR;
     static constexpr int NCH = DPL / 8;
     static constexpr int STEPS = TR / RPS;
-    static constexpr int NSUM = (TR * G + 31) / 32;
-    static constexpr int GP = G <= 4 ? 4 : 8;  // p row stride (floats)
-    // Reduction buffer red[j][r][step][s]: RS is the r stride, = LPR (mod 32), so
-    // the 32 lanes of one store (fixed j, step) hit 32 distinct banks.
-    static constexpr int RS0 = STEPS * LPR;
-    static constexpr int RS = RS0 + ((LPR - RS0 % 32) + 32) % 32;
-    static constexpr int JS = RPS * RS;
-    static constexpr int kRedFloats = G * JS;
-    static constexpr int kPFloats = TR * GP;
-    static constexpr int kWarpScratch = (kRedFloats + kPFloats) * 4;
+    static constexpr int HPU = 32 / TR;  // heads per score slot index u
+    static constexpr int NSUM = (G + HPU - 1) / HPU;
+    static constexpr int GP = G <= 4 ? 4 : 8;  // p pairs per row in shared memory
+    // Reduction buffer red[j][step][r][sl]: the 32 lanes of one store (fixed j,
+    // step) write 32 consecutive floats; a score sums LPR consecutive floats.
+    // The p pairs of a tile reuse the same bytes once the scores are read.
+    static constexpr int kRedFloats = G * STEPS * 32;
+    static constexpr int kPFloats = TR * GP * 2;
+    static constexpr int kWarpScratch = ((kRedFloats > kPFloats ? kRedFloats : kPFloats) * 4 + 15) / 16 * 16;
     static constexpr int kStageBytes = 2 * TR * kRowBytes;  // K tile then V tile
     static constexpr int kRingBytes = NW * NS * kStageBytes;
-    static constexpr int kMergeBytes = NW * G * (kHeadDim + 2) * 4;
-    static constexpr int kScratchBytes = (NW * kWarpScratch > kMergeBytes) ? NW * kWarpScratch : kMergeBytes;
+    static constexpr int kScratchBytes = NW * kWarpScratch;
     static constexpr int kBarBytes = NW * NS * 8;
-    static constexpr int kFixedBytes = kRingBytes + kScratchBytes + kBarBytes;
+    static constexpr int kMetaBytes = NW * 2 * 4 + 16;  // first/last slab of each warp
+    static constexpr int kFixedBytes = kRingBytes + kScratchBytes + kBarBytes + kMetaBytes;
+    static constexpr int kStateFloats = G * (kHeadDim + 2);
     static int bytes(int B) { return kFixedBytes + (2 * B + 1) * 4; }
     static_assert(TR % RPS == 0 && 32 % TR == 0, "tile geometry");
-    static_assert(RS % 4 == 0, "16-byte aligned reduction rows");
+    static_assert(kStateFloats * 4 <= NS * kStageBytes, "a warp's final state fits in its ring");
 };
 
-// Tile cursor of one warp over the CTA's slab segments, with the segment's
-// constants cached (slab start row in the cache, rows, append flag).
+// Tile cursor of one warp over its row range, with the current slab's constants.
 struct Cursor {
-    int h;        // slab; == hend when exhausted
-    int64_t s0;   // segment global rows [s0, s1)
-    int64_t s1;
-    int64_t p0;   // slab_start(h)
-    int64_t base; // off[h]: first cache row of the slab
-    int n_h;      // rows of the slab in this call
-    int app;      // this call appends the slab's last row from k_new/v_new
-    int t;        // tile index within the segment
+    int h;         // slab; == hend when exhausted
+    int s0, s1;    // the warp's rows of this slab, [s0, s1) (layer rows)
+    int p0;        // slab_start(h)
+    int x;         // first row of the current tile
+    int n_h;       // rows of the slab in this call
+    int app;       // this call appends the slab's last row from k_new/v_new
+    int64_t base;  // off[h]: cache row of the slab's first row
 };
 
-template <int TR, int NW>
-__device__ __forceinline__ void cursor_seek(Cursor& cu, const DecodeArgs& a, const SeqTable& t,
-                                            int hend, int64_t A, int64_t Bc, int warp)
+__device__ __forceinline__ void cursor_seek(Cursor& cu, const DecodeArgs& a, const SeqTable& t, int hend, int wA,
+                                            int wB)
 {
-    // Advance from cu.h (inclusive) to the first slab whose segment has a tile for `warp`.
     while (cu.h < hend) {
         cu.p0 = slab_start(a, t, cu.h);
-        const int64_t p1 = slab_start(a, t, cu.h + 1);
-        cu.s0 = max(A, cu.p0);
-        cu.s1 = min(Bc, p1);
-        cu.t = warp;
-        if (cu.s0 + (int64_t)warp * TR < cu.s1) {
+        const int p1 = slab_start(a, t, cu.h + 1);
+        cu.s0 = max(wA, cu.p0);
+        cu.s1 = min(wB, p1);
+        if (cu.s0 < cu.s1) {
             const int b = cu.h / a.Hkv;
             const int e = t.NP[b + 1] - t.NP[b];
             cu.n_h = a.len[cu.h] + e;
             cu.app = (a.append && e > t.NA[b]) ? 1 : 0;
             cu.base = a.off[cu.h];
+            cu.x = cu.s0;
             return;
         }
         ++cu.h;
     }
 }
 
-template <int TR, int NW>
-__device__ __forceinline__ void cursor_next(Cursor& cu, const DecodeArgs& a, const SeqTable& t,
-                                            int hend, int64_t A, int64_t Bc, int warp)
+template <int TR>
+__device__ __forceinline__ void cursor_next(Cursor& cu, const DecodeArgs& a, const SeqTable& t, int hend, int wA,
+                                            int wB)
 {
-    cu.t += NW;
-    if (cu.s0 + (int64_t)cu.t * TR < cu.s1) return;
+    cu.x += TR;
+    if (cu.x < cu.s1) return;
     ++cu.h;
-    cursor_seek<TR, NW>(cu, a, t, hend, A, Bc, warp);
+    cursor_seek(cu, a, t, hend, wA, wB);
 }
 
+// Per-warp running state of one slab segment.
 template <class C>
-__global__ void __launch_bounds__(C::NW * 32, 1) decode_partial_kernel(const DecodeArgs a)
+struct State {
+    float m_all[C::G];       // running max per head (log2 domain), same in every lane
+    float m_my[C::NSUM];     // running max of the heads of the lane's score slots
+    float l_my[C::NSUM];     // the lane's share of the softmax denominator
+    uint64_t o2[C::G][C::DPL / 2];  // unnormalised output, the lane's dims of its rows
+};
+
+// One tile: scores, online softmax, o += p v. FULL: all TR rows are valid.
+template <class C, bool FULL>
+__device__ __forceinline__ void tile_compute(State<C>& S, const uint64_t (&q2)[C::G][C::DPL / 2],
+                                             const unsigned char* kt, const unsigned char* vt, float* red,
+                                             float2* ps, int cnt, float cs, int lane)
 {
-    constexpr int G = C::G, LPR = C::LPR, TR = C::TR, NS = C::NS, NW = C::NW;
-    constexpr int RPS = C::RPS, DPL = C::DPL, NCH = C::NCH, STEPS = C::STEPS, NSUM = C::NSUM;
-    extern __shared__ __align__(128) unsigned char smem[];
-    unsigned char* ring = smem;
-    unsigned char* scratch = smem + C::kRingBytes;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(scratch + C::kScratchBytes);
-    SeqTable tab;
-    tab.NA = reinterpret_cast<int32_t*>(smem + C::kFixedBytes);
-    tab.NP = tab.NA + a.B;
+    constexpr int G = C::G, LPR = C::LPR, TR = C::TR, RPS = C::RPS, DPL = C::DPL, NCH = C::NCH;
+    constexpr int STEPS = C::STEPS, NSUM = C::NSUM, HPU = C::HPU;
+    const int r = lane / LPR, sl = lane % LPR;
 
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int r = lane / LPR, sl = lane % LPR;  // row within a step, dim slice
-    const int NHl = a.B * a.Hkv;
-    const int c = blockIdx.x;
-
-    if (warp == 0) build_seq_table(a, tab, c == 0);
-    if (lane == 0) {
-        for (int s = 0; s < NS; ++s) mbar_init(smem_u32(&bars[warp * NS + s]), 1);
-        fence_proxy_async_smem();
-    }
-    __syncthreads();
-
-    const int64_t R = slab_start(a, tab, NHl);
-    if (R == 0) return;
-    const int64_t A = cta_start(c, R, a.nctas), Bc = cta_start(c + 1, R, a.nctas);
-    if (A >= Bc) return;
-    const int hfirst = slab_containing(a, tab, NHl, A);
-    const int hend = slab_containing(a, tab, NHl, Bc - 1) + 1;
-
-    const uint64_t pol = evict_first_policy();
-    unsigned char* my_ring = ring + warp * NS * C::kStageBytes;
-    uint64_t* my_bars = bars + warp * NS;
-    float* red = reinterpret_cast<float*>(scratch + warp * C::kWarpScratch);
-    float* ps = red + C::kRedFloats;
-    float* mrg = reinterpret_cast<float*>(scratch);
-
-    Cursor ld{hfirst, 0, 0, 0, 0, 0, 0, 0};
-    cursor_seek<TR, NW>(ld, a, tab, hend, A, Bc, warp);
-    Cursor cp = ld;
-
-    auto issue = [&](const Cursor& cu, int stage) {
-        const int64_t x0 = cu.s0 + (int64_t)cu.t * TR;
-        const int cnt = (int)min((int64_t)TR, cu.s1 - x0);
-        const int r0 = (int)(x0 - cu.p0);
-        const int ncopy = (cu.app && r0 + cnt == cu.n_h) ? cnt - 1 : cnt;  // new token comes from k_new
-        const uint32_t bar = smem_u32(&my_bars[stage]);
-        unsigned char* dst = my_ring + stage * C::kStageBytes;
-        const uint32_t bytes = (uint32_t)ncopy * kRowBytes;
-        fence_proxy_async_smem();
-        mbar_arrive_expect_tx(bar, 2 * bytes);
-        if (ncopy > 0) {
-            const int64_t row = cu.base + r0;
-            bulk_g2s(smem_u32(dst), a.Kc + row * kHeadDim, bytes, bar, pol);
-            bulk_g2s(smem_u32(dst + TR * kRowBytes), a.Vc + row * kHeadDim, bytes, bar, pol);
-        }
-    };
-
-    bool dead = false;
-    int inflight = 0;
-    int dead_stage = 0, dead_inflight = 0;
-    uint32_t dead_phase = 0;
-    if (lane == 0) {
-        Cursor it = ld;
-        for (int s = 0; s < NS && it.h < hend; ++s) {
-            issue(it, s);
-            cursor_next<TR, NW>(it, a, tab, hend, A, Bc, warp);
-        }
-    }
-    for (int s = 0; s < NS && ld.h < hend; ++s) {
-        ++inflight;
-        cursor_next<TR, NW>(ld, a, tab, hend, A, Bc, warp);
-    }
-    int stage = 0;
-    uint32_t phase = 0;
-    const float cs = a.qscale;  // softmax scale * log2(e)
-
-    for (int h = hfirst; h < hend; ++h) {
-        {
-            const int64_t p0 = slab_start(a, tab, h), p1 = slab_start(a, tab, h + 1);
-            if (max(A, p0) >= min(Bc, p1)) continue;  // empty slab: nothing to merge (uniform)
-        }
-        const int b = h / a.Hkv, g = h - b * a.Hkv;
-        // q of the group, unscaled, as packed fp32 pairs of the lane's dims.
-        uint64_t q2[G][DPL / 2];
+    // q.k partial sums over the lane's dims -> red[j][step][r][sl].
+#pragma unroll
+    for (int st = 0; st < STEPS; ++st) {
+        const int row = st * RPS + r;
+        uint64_t k2[DPL / 2];
+#pragma unroll
+        for (int i = 0; i < NCH; ++i)
+            bf8_to_f2x4(*reinterpret_cast<const uint4*>(kt + row * kRowBytes + 16 * (sl + LPR * i)), k2 + 4 * i);
 #pragma unroll
         for (int j = 0; j < G; ++j) {
-            const uint16_t* qrow = a.q + ((int64_t)b * a.H + g * G + j) * kHeadDim;
+            uint64_t acc = mul2(q2[j][0], k2[0]);
 #pragma unroll
-            for (int i = 0; i < NCH; ++i) {
-                const uint4 w = *reinterpret_cast<const uint4*>(qrow + 8 * (sl + LPR * i));
-                q2[j][4 * i + 0] = bf2_to_f2(w.x);
-                q2[j][4 * i + 1] = bf2_to_f2(w.y);
-                q2[j][4 * i + 2] = bf2_to_f2(w.z);
-                q2[j][4 * i + 3] = bf2_to_f2(w.w);
+            for (int i = 1; i < DPL / 2; ++i) acc = fma2(q2[j][i], k2[i], acc);
+            const float2 f = upk(acc);
+            red[(j * STEPS + st) * 32 + lane] = f.x + f.y;
+        }
+    }
+    __syncwarp();
+    // Full scores of the lane's slots.
+    const int row = lane % TR;
+    float sc[NSUM];
+#pragma unroll
+    for (int u = 0; u < NSUM; ++u) {
+        const int j = lane / TR + u * HPU;
+        float v = -INFINITY;
+        if (NSUM * HPU == G || j < G) {
+            const float4* src = reinterpret_cast<const float4*>(red + (j * STEPS + row / RPS) * 32 +
+                                                                 (row % RPS) * LPR);
+            float4 acc = src[0];
+#pragma unroll
+            for (int i = 1; i < LPR / 4; ++i) {
+                const float4 x = src[i];
+                acc.x += x.x;
+                acc.y += x.y;
+                acc.z += x.z;
+                acc.w += x.w;
             }
+            v = (acc.x + acc.y) + (acc.z + acc.w);
+            if (!FULL && row >= cnt) v = -INFINITY;
         }
-        // Running state: m per head (same in every lane), the lane's share of l
-        // for its score slots, o for its dims of its rows.
-        float m_all[G], m_my[NSUM], l_my[NSUM];
-        uint64_t o2[G][DPL / 2];
+        sc[u] = v;
+    }
+    // Lazy rescaling: the running max m of a head only moves when a score tops it
+    // by more than kSlack (log2 units), so p = 2^(s - m) <= 2^kSlack and most tiles
+    // need one vote instead of a cross-lane max. The first tile always moves m.
+    bool over = false;
+#pragma unroll
+    for (int u = 0; u < NSUM; ++u) over |= sc[u] * cs > S.m_my[u] + kSlack;
+    if (__any_sync(kFull, over)) {
+        float mnew_my[NSUM];
+#pragma unroll
+        for (int u = 0; u < NSUM; ++u) {
+            float x = sc[u];
+#pragma unroll
+            for (int o = TR / 2; o >= 1; o >>= 1) x = fmaxf(x, __shfl_xor_sync(kFull, x, o));
+            mnew_my[u] = fmaxf(S.m_my[u], x * cs);
+        }
 #pragma unroll
         for (int j = 0; j < G; ++j) {
-            m_all[j] = -INFINITY;
+            const float mn = __shfl_sync(kFull, mnew_my[j / HPU], (j % HPU) * TR);
+            const float al = (mn == -INFINITY) ? 1.f : ex2(S.m_all[j] - mn);
+            const uint64_t al2 = pk(al, al);
 #pragma unroll
-            for (int i = 0; i < DPL / 2; ++i) o2[j][i] = 0ull;
+            for (int i = 0; i < DPL / 2; ++i) S.o2[j][i] = mul2(S.o2[j][i], al2);
+            S.m_all[j] = mn;
         }
 #pragma unroll
         for (int u = 0; u < NSUM; ++u) {
-            m_my[u] = -INFINITY;
-            l_my[u] = 0.f;
+            S.l_my[u] *= (mnew_my[u] == -INFINITY) ? 1.f : ex2(S.m_my[u] - mnew_my[u]);
+            S.m_my[u] = mnew_my[u];
         }
+    }
+    __syncwarp();  // the p pairs below overwrite the reduction buffer
+#pragma unroll
+    for (int u = 0; u < NSUM; ++u) {
+        const int j = lane / TR + u * HPU;
+        const float mref = (S.m_my[u] == -INFINITY) ? 0.f : S.m_my[u];
+        const float p = ex2(fmaf(sc[u], cs, -mref));  // exp2(-inf) = 0 for masked rows
+        S.l_my[u] += p;
+        if (NSUM * HPU == G || j < G) ps[row * C::GP + j] = make_float2(p, p);
+    }
+    __syncwarp();
+    // o += p v over the lane's dims.
+#pragma unroll
+    for (int st = 0; st < STEPS; ++st) {
+        const int vrow = st * RPS + r;
+        uint64_t pp[C::GP];
+#pragma unroll
+        for (int q4 = 0; q4 < C::GP / 2; ++q4) {
+            const ulonglong2 w = *reinterpret_cast<const ulonglong2*>(ps + vrow * C::GP + 2 * q4);
+            pp[2 * q4] = w.x;
+            pp[2 * q4 + 1] = w.y;
+        }
+        uint64_t v2[DPL / 2];
+#pragma unroll
+        for (int i = 0; i < NCH; ++i) {
+            uint4 w = *reinterpret_cast<const uint4*>(vt + vrow * kRowBytes + 16 * (sl + LPR * i));
+            if (!FULL && vrow >= cnt) w = make_uint4(0u, 0u, 0u, 0u);  // stale bytes may not be finite
+            bf8_to_f2x4(w, v2 + 4 * i);
+        }
+#pragma unroll
+        for (int j = 0; j < G; ++j)
+#pragma unroll
+            for (int i = 0; i < DPL / 2; ++i) S.o2[j][i] = fma2(pp[j], v2[i], S.o2[j][i]);
+    }
+}
 
-        while (cp.h == h) {
-            const int64_t x0 = cp.s0 + (int64_t)cp.t * TR;
-            const int cnt = (int)min((int64_t)TR, cp.s1 - x0);
-            const int r0 = (int)(x0 - cp.p0);
-            unsigned char* kt = my_ring + stage * C::kStageBytes;
-            unsigned char* vt = kt + TR * kRowBytes;
-            if (!dead) {
-                const bool ok = __all_sync(kFull, mbar_wait(smem_u32(&my_bars[stage]), phase));
-                if (ok) {
-                    --inflight;
-                } else {
-                    dead = true;
-                    dead_stage = stage;
-                    dead_phase = phase;
-                    dead_inflight = inflight;
-                    if (lane == 0) atomicOr(a.status, 0x2 /* DKV_DEV_TMA_TIMEOUT */);
-                }
+// Number of CTAs whose row range overlaps [p0, p1) (p0 < p1), and the first and
+// last of them.
+__device__ __forceinline__ int ctas_of_slab(int p0, int p1, int R, int P, int* c0_out, int* c1_out)
+{
+    const int c0 = part_of(p0, R, P), c1 = part_of(p1 - 1, R, P);
+    int n = c1 - c0 + 1;
+    if (R < P) {  // some CTAs have no rows (never when every CTA gets at least one)
+        n = 0;
+        for (int cc = c0; cc <= c1; ++cc) n += part_start(cc, R, P) < part_start(cc + 1, R, P) ? 1 : 0;
+    }
+    *c0_out = c0;
+    *c1_out = c1;
+    return n;
+}
+
+// out[b][g*G + j] = O / L for the group's heads; O, L per head j for the lane's 4 dims.
+template <int G>
+__device__ __forceinline__ void write_out(const DecodeArgs& a, int b, int g, int j, float4 O, float L, int lane)
+{
+    const float inv = L > 0.f ? 1.f / L : 0.f;
+    float4* dst = reinterpret_cast<float4*>(a.out + ((int64_t)b * a.H + g * G + j) * kHeadDim);
+    dst[lane] = make_float4(O.x * inv, O.y * inv, O.z * inv, O.w * inv);
+}
+
+// Fused combine of head j of slab h by one warp of the last CTA to finish the
+// slab: the CTA partials in slots c + h, c in [c0, c1]. Lanes read the (m, l) of
+// 32 partials at a time in parallel; the weighted sum of o then loads four
+// partials at a time, all four loads in flight before any is used. Partials come
+// from other SMs: L2 loads.
+template <int G>
+__device__ void merge_slab_head(const DecodeArgs& a, int h, int j, int c0, int c1, int R, int lane)
+{
+    const int b = h / a.Hkv, g = h - b * a.Hkv;
+    const int n = c1 - c0 + 1;
+    const int P = a.nctas;
+    const bool all_live = R >= P;  // every CTA has rows
+    auto live = [&](int cc) { return all_live || part_start(cc, R, P) < part_start(cc + 1, R, P); };
+    float M = -INFINITY;
+    for (int base = 0; base < n; base += 32) {
+        const int cc = c0 + base + lane;
+        if (base + lane < n && live(cc)) M = fmaxf(M, __ldcg(a.work_ml + (((int64_t)cc + h) * G + j) * 2));
+    }
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) M = fmaxf(M, __shfl_xor_sync(kFull, M, o));
+    float L = 0.f;
+    float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int base = 0; base < n; base += 32) {
+        const int cc = c0 + base + lane;
+        float f = 0.f;
+        if (base + lane < n && live(cc)) {
+            const float2 ml = __ldcg(reinterpret_cast<const float2*>(a.work_ml + (((int64_t)cc + h) * G + j) * 2));
+            f = (ml.x == -INFINITY) ? 0.f : ex2(ml.x - M);
+            L = fmaf(f, ml.y, L);
+        }
+        const int cnt = min(32, n - base);
+        for (int k0 = 0; k0 < cnt; k0 += 4) {
+            float fk[4];
+            float4 v[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) fk[u] = __shfl_sync(kFull, f, (k0 + u) & 31);
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int ck = c0 + base + k0 + u;
+                v[u] = (k0 + u < cnt && live(ck))
+                           ? __ldcg(reinterpret_cast<const float4*>(a.work_o + (((int64_t)ck + h) * G + j) * kHeadDim) + lane)
+                           : make_float4(0.f, 0.f, 0.f, 0.f);
             }
-            if (!dead) {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const float w = (k0 + u < cnt) ? fk[u] : 0.f;
+                O.x = fmaf(w, v[u].x, O.x);
+                O.y = fmaf(w, v[u].y, O.y);
+                O.z = fmaf(w, v[u].z, O.z);
+                O.w = fmaf(w, v[u].w, O.w);
+            }
+        }
+    }
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) L += __shfl_xor_sync(kFull, L, o);
+    write_out<G>(a, b, g, j, O, L, lane);
+}
+
+// Final answer of a slab held by one warp: out = o / l for the lane's dims
+// (lanes with r == 0 hold o after finish_state).
+template <class C>
+__device__ __forceinline__ void write_out_state(const DecodeArgs& a, const State<C>& S, const float (&l_all)[C::G],
+                                                int b, int g, int lane)
+{
+    constexpr int G = C::G, LPR = C::LPR, NCH = C::NCH;
+    const int r = lane / LPR, sl = lane % LPR;
+    if (r != 0) return;
+#pragma unroll
+    for (int j = 0; j < G; ++j) {
+        const float inv = l_all[j] > 0.f ? 1.f / l_all[j] : 0.f;
+        float* dst = a.out + ((int64_t)b * a.H + g * G + j) * kHeadDim;
+#pragma unroll
+        for (int i = 0; i < NCH; ++i) {
+            float4* d = reinterpret_cast<float4*>(dst + 8 * (sl + LPR * i));
+            const float2 a0 = upk(S.o2[j][4 * i + 0]), a1 = upk(S.o2[j][4 * i + 1]);
+            const float2 a2 = upk(S.o2[j][4 * i + 2]), a3 = upk(S.o2[j][4 * i + 3]);
+            d[0] = make_float4(a0.x * inv, a0.y * inv, a1.x * inv, a1.y * inv);
+            d[1] = make_float4(a2.x * inv, a2.y * inv, a3.x * inv, a3.y * inv);
+        }
+    }
+}
+
+// Writes a warp state (o over the lane's dims for the RPS row lanes already
+// summed, m and l per head) as one record: o[G][128] at o_dst, (m, l)[G] at ml_dst.
+template <class C>
+__device__ __forceinline__ void store_state(const State<C>& S, const float (&l_all)[C::G], float* o_dst,
+                                            float* ml_dst, int lane)
+{
+    constexpr int G = C::G, LPR = C::LPR, NCH = C::NCH;
+    const int r = lane / LPR, sl = lane % LPR;
+    if (r == 0) {
+#pragma unroll
+        for (int j = 0; j < G; ++j)
+#pragma unroll
+            for (int i = 0; i < NCH; ++i) {
+                float4* d = reinterpret_cast<float4*>(o_dst + j * kHeadDim + 8 * (sl + LPR * i));
+                const float2 a0 = upk(S.o2[j][4 * i + 0]), a1 = upk(S.o2[j][4 * i + 1]);
+                const float2 a2 = upk(S.o2[j][4 * i + 2]), a3 = upk(S.o2[j][4 * i + 3]);
+                d[0] = make_float4(a0.x, a0.y, a1.x, a1.y);
+                d[1] = make_float4(a2.x, a2.y, a3.x, a3.y);
+            }
+    }
+    if (lane == 0) {
+#pragma unroll
+        for (int j = 0; j < G; ++j) *reinterpret_cast<float2*>(ml_dst + 2 * j) = make_float2(S.m_all[j], l_all[j]);
+    }
+}
+
+// Sums a segment's state over the RPS row lanes (o) and the TR lanes of each
+// head (l); afterwards lanes with r == 0 hold o of their dims, l_all is per head.
+template <class C>
+__device__ __forceinline__ void finish_state(State<C>& S, float (&l_all)[C::G])
+{
+    constexpr int G = C::G, LPR = C::LPR, TR = C::TR, DPL = C::DPL, NSUM = C::NSUM, HPU = C::HPU;
+#pragma unroll
+    for (int o = LPR; o < 32; o <<= 1)
+#pragma unroll
+        for (int j = 0; j < G; ++j)
+#pragma unroll
+            for (int i = 0; i < DPL / 2; ++i) {
+                const float2 f = upk(S.o2[j][i]);
+                S.o2[j][i] = add2(S.o2[j][i], pk(__shfl_xor_sync(kFull, f.x, o), __shfl_xor_sync(kFull, f.y, o)));
+            }
+#pragma unroll
+    for (int u = 0; u < NSUM; ++u) {
+        float x = S.l_my[u];
+#pragma unroll
+        for (int o = TR / 2; o >= 1; o >>= 1) x += __shfl_xor_sync(kFull, x, o);
+        S.l_my[u] = x;
+    }
+#pragma unroll
+    for (int j = 0; j < G; ++j) l_all[j] = __shfl_sync(kFull, S.l_my[j / HPU], (j % HPU) * TR);
+}
+
+template <class C, bool FUSED>
+__global__ void __launch_bounds__(C::NW * 32, 1) decode_partial_kernel(const DecodeArgs a)
+{
+    constexpr int G = C::G, LPR = C::LPR, TR = C::TR, NS = C::NS, NW = C::NW;
+    constexpr int DPL = C::DPL, NCH = C::NCH, NSUM = C::NSUM;
+    extern __shared__ __align__(128) unsigned char smem[];
+    SeqTable tab;
+    tab.NA = reinterpret_cast<int32_t*>(smem + C::kFixedBytes);
+    tab.NP = tab.NA + a.B;
+    int32_t* seg_first = reinterpret_cast<int32_t*>(smem + C::kRingBytes + C::kScratchBytes + C::kBarBytes);
+    int32_t* seg_last = seg_first + NW;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int sl = lane % LPR;
+    const int NHl = a.B * a.Hkv;
+    const int c = blockIdx.x;
+    uint64_t* my_bars = reinterpret_cast<uint64_t*>(smem + C::kRingBytes + C::kScratchBytes) + warp * NS;
+
+    if (warp == 0) build_seq_table(a, tab, c == 0);
+    if (lane == 0) {
+        for (int s = 0; s < NS; ++s) mbar_init(smem_u32(&my_bars[s]), 1);
+        fence_proxy_async_smem();
+        seg_first[warp] = -1;
+        seg_last[warp] = -1;
+    }
+    __syncthreads();  // table, barriers and slab entries are ready
+    pdl_launch_dependents();
+
+    const int R = slab_start(a, tab, NHl);
+    if (FUSED && c == a.nctas - 1 && warp == 0) {
+        // Slabs with no rows belong to no CTA: their outputs are zero (written by
+        // the last CTA, which always runs; after the wait, as any write of out).
+        pdl_wait();
+        for (int h = 0; h < NHl; ++h)
+            if (slab_start(a, tab, h) == slab_start(a, tab, h + 1))
+                for (int j = 0; j < G; ++j)
+                    write_out<G>(a, h / a.Hkv, h % a.Hkv, j, make_float4(0.f, 0.f, 0.f, 0.f), 0.f, lane);
+    }
+    const int A = part_start(c, R, a.nctas), Bc = part_start(c + 1, R, a.nctas);
+    if (A >= Bc) return;  // uniform: this CTA has no rows
+    const int wA = A + (int)(((int64_t)(Bc - A) * warp) / NW);
+    const int wB = A + (int)(((int64_t)(Bc - A) * (warp + 1)) / NW);
+    unsigned char* my_ring = smem + warp * NS * C::kStageBytes;
+    State<C> S;
+    float l_all[G];
+    bool have_last = false;  // S holds the state of this warp's last slab
+
+    if (wA < wB) {
+        const int hfirst = slab_containing(a, tab, NHl, wA);
+        const int hlast = slab_containing(a, tab, NHl, wB - 1);
+        const int hend = hlast + 1;
+        const uint64_t pol = evict_first_policy();
+        float* red = reinterpret_cast<float*>(smem + C::kRingBytes + warp * C::kWarpScratch);
+        float2* ps = reinterpret_cast<float2*>(red);
+
+        Cursor ld;
+        ld.h = hfirst;
+        cursor_seek(ld, a, tab, hend, wA, wB);
+        Cursor cp = ld;
+
+        auto issue = [&](const Cursor& cu, int stage) {
+            const int cnt = min(TR, cu.s1 - cu.x);
+            const int r0 = cu.x - cu.p0;  // row within the slab
+            const int ncopy = (cu.app && r0 + cnt == cu.n_h) ? cnt - 1 : cnt;  // new token comes from k_new
+            const uint32_t bar = smem_u32(&my_bars[stage]);
+            unsigned char* dst = my_ring + stage * C::kStageBytes;
+            const uint32_t bytes = (uint32_t)ncopy * kRowBytes;
+            fence_proxy_async_smem();
+            mbar_arrive_expect_tx(bar, 2 * bytes);
+            if (ncopy > 0) {
+                const int64_t row = cu.base + r0;
+                bulk_g2s(smem_u32(dst), a.Kc + row * kHeadDim, bytes, bar, pol);
+                bulk_g2s(smem_u32(dst + TR * kRowBytes), a.Vc + row * kHeadDim, bytes, bar, pol);
+            }
+        };
+
+        // A bounded wait that runs out marks the warp dead: it stops issuing and
+        // computing, drains its copies in flight, and leaves its partials unwritten.
+        bool dead = false;
+        int inflight = 0;
+        if (lane == 0) {
+            Cursor it = ld;
+            for (int s = 0; s < NS && it.h < hend; ++s) {
+                issue(it, s);
+                cursor_next<TR>(it, a, tab, hend, wA, wB);
+            }
+        }
+        for (int s = 0; s < NS && ld.h < hend; ++s) {
+            ++inflight;
+            cursor_next<TR>(ld, a, tab, hend, wA, wB);
+        }
+        // Everything above reads only the plan, n_appended and the cache rows of
+        // earlier steps; q, k_new, v_new, the cache slots written here and the
+        // workspace belong to the previous kernel's epoch.
+        pdl_wait();
+        int stage = 0;
+        uint32_t phase = 0;
+        const float cs = a.qscale;  // softmax scale * log2(e)
+
+        while (cp.h < hend && !dead) {
+            const int h = cp.h;
+            const int b = h / a.Hkv, g = h - b * a.Hkv;
+            // q of the group, unscaled, as packed fp32 pairs of the lane's dims.
+            uint64_t q2[G][DPL / 2];
+#pragma unroll
+            for (int j = 0; j < G; ++j) {
+                const uint16_t* qrow = a.q + ((int64_t)b * a.H + g * G + j) * kHeadDim;
+#pragma unroll
+                for (int i = 0; i < NCH; ++i)
+                    bf8_to_f2x4(__ldg(reinterpret_cast<const uint4*>(qrow + 8 * (sl + LPR * i))), q2[j] + 4 * i);
+            }
+#pragma unroll
+            for (int j = 0; j < G; ++j) {
+                S.m_all[j] = -INFINITY;
+#pragma unroll
+                for (int i = 0; i < DPL / 2; ++i) S.o2[j][i] = 0ull;
+            }
+#pragma unroll
+            for (int u = 0; u < NSUM; ++u) {
+                S.m_my[u] = -INFINITY;
+                S.l_my[u] = 0.f;
+            }
+
+            while (cp.h == h) {
+                const int cnt = min(TR, cp.s1 - cp.x);
+                const int r0 = cp.x - cp.p0;
+                unsigned char* kt = my_ring + stage * C::kStageBytes;
+                unsigned char* vt = kt + TR * kRowBytes;
+                // Every lane observes the completed phase itself (acquire) before reading.
+                if (!__all_sync(kFull, mbar_wait(smem_u32(&my_bars[stage]), phase))) {
+                    dead = true;
+                    if (lane == 0) atomicOr(a.status, 0x2 /* DKV_DEV_TMA_TIMEOUT */);
+                    break;
+                }
+                --inflight;
                 if (cp.app && r0 + cnt == cp.n_h) {
                     // This step's token: into the tile from k_new/v_new, and into the
                     // slab's next free row for later steps.
                     const int half = lane >> 4, sub = lane & 15;
-                    const int rr = cnt - 1;
                     const uint16_t* src = (half ? a.v_new : a.k_new) + ((int64_t)b * a.Hkv + g) * kHeadDim;
-                    const uint4 v = *(reinterpret_cast<const uint4*>(src) + sub);
-                    *reinterpret_cast<uint4*>((half ? vt : kt) + rr * kRowBytes + sub * 16) = v;
+                    const uint4 v = __ldg(reinterpret_cast<const uint4*>(src) + sub);
+                    *reinterpret_cast<uint4*>((half ? vt : kt) + (cnt - 1) * kRowBytes + sub * 16) = v;
                     uint16_t* dstg = (half ? a.Vc : a.Kc) + (cp.base + (cp.n_h - 1)) * kHeadDim;
                     *(reinterpret_cast<uint4*>(dstg) + sub) = v;
                     fence_proxy_async_smem();  // order these generic writes before later bulk copies
                     __syncwarp();
                 }
-
-                // q.k partial sums over the lane's dims -> red[j][r][step][sl].
-#pragma unroll
-                for (int st = 0; st < STEPS; ++st) {
-                    const int row = st * RPS + r;
-                    uint64_t k2[DPL / 2];
-#pragma unroll
-                    for (int i = 0; i < NCH; ++i) {
-                        const uint4 w = *reinterpret_cast<const uint4*>(kt + row * kRowBytes + 16 * (sl + LPR * i));
-                        k2[4 * i + 0] = bf2_to_f2(w.x);
-                        k2[4 * i + 1] = bf2_to_f2(w.y);
-                        k2[4 * i + 2] = bf2_to_f2(w.z);
-                        k2[4 * i + 3] = bf2_to_f2(w.w);
-                    }
-#pragma unroll
-                    for (int j = 0; j < G; ++j) {
-                        uint64_t acc = mul2(q2[j][0], k2[0]);
-#pragma unroll
-                        for (int i = 1; i < DPL / 2; ++i) acc = fma2(q2[j][i], k2[i], acc);
-                        const float2 f = upk(acc);
-                        red[j * C::JS + r * C::RS + st * LPR + sl] = f.x + f.y;
-                    }
-                }
+                if (cnt == TR)
+                    tile_compute<C, true>(S, q2, kt, vt, red, ps, cnt, cs, lane);
+                else
+                    tile_compute<C, false>(S, q2, kt, vt, red, ps, cnt, cs, lane);
                 __syncwarp();
-                // Full scores of the lane's slots: slot k = lane + 32u -> (row k % TR, head k / TR).
-                float sc[NSUM];
-#pragma unroll
-                for (int u = 0; u < NSUM; ++u) {
-                    const int k = lane + 32 * u;
-                    const int row = k % TR, j = k / TR;
-                    float v = -INFINITY;
-                    if (j < G) {
-                        const float4* src = reinterpret_cast<const float4*>(
-                            red + j * C::JS + (row % RPS) * C::RS + (row / RPS) * LPR);
-                        float4 acc = src[0];
-#pragma unroll
-                        for (int i = 1; i < LPR / 4; ++i) {
-                            const float4 x = src[i];
-                            acc.x += x.x;
-                            acc.y += x.y;
-                            acc.z += x.z;
-                            acc.w += x.w;
-                        }
-                        const float d = (acc.x + acc.y) + (acc.z + acc.w);
-                        if (row < cnt) v = d;
-                    }
-                    sc[u] = v;
+                // Refill this stage with the tile NS ahead.
+                if (ld.h < hend) {
+                    if (lane == 0) issue(ld, stage);
+                    ++inflight;
+                    cursor_next<TR>(ld, a, tab, hend, wA, wB);
                 }
-                // Tile max per head (over the TR lanes that hold that head), then
-                // the new running max of every head in every lane.
-                float mnew_my[NSUM];
-#pragma unroll
-                for (int u = 0; u < NSUM; ++u) {
-                    float x = sc[u];
-#pragma unroll
-                    for (int o = TR / 2; o >= 1; o >>= 1) x = fmaxf(x, __shfl_xor_sync(kFull, x, o));
-                    mnew_my[u] = fmaxf(m_my[u], x * cs);
-                }
-                float mnew_all[G];
-                bool grow = false;
-#pragma unroll
-                for (int j = 0; j < G; ++j) {
-                    mnew_all[j] = __shfl_sync(kFull, mnew_my[(j * TR) / 32], (j * TR) % 32);
-                    grow |= mnew_all[j] > m_all[j];
-                }
-                if (__any_sync(kFull, grow)) {  // rare after the first tiles
-#pragma unroll
-                    for (int j = 0; j < G; ++j) {
-                        const float al = (mnew_all[j] == -INFINITY) ? 1.f : ex2(m_all[j] - mnew_all[j]);
-                        const uint64_t al2 = pk(al, al);
-#pragma unroll
-                        for (int i = 0; i < DPL / 2; ++i) o2[j][i] = mul2(o2[j][i], al2);
-                        m_all[j] = mnew_all[j];
-                    }
-#pragma unroll
-                    for (int u = 0; u < NSUM; ++u)
-                        l_my[u] *= (mnew_my[u] == -INFINITY) ? 1.f : ex2(m_my[u] - mnew_my[u]);
-                }
-#pragma unroll
-                for (int u = 0; u < NSUM; ++u) {
-                    m_my[u] = mnew_my[u];
-                    const int k = lane + 32 * u;
-                    const int row = k % TR, j = k / TR;
-                    const float p = (sc[u] == -INFINITY) ? 0.f : ex2(fmaf(sc[u], cs, -m_my[u]));
-                    l_my[u] += p;
-                    if (j < G) ps[row * C::GP + j] = p;
-                }
-                __syncwarp();
-                // o += p v over the lane's dims.
-#pragma unroll
-                for (int st = 0; st < STEPS; ++st) {
-                    const int row = st * RPS + r;
-                    float pj[C::GP];
-#pragma unroll
-                    for (int q4 = 0; q4 < C::GP / 4; ++q4) {
-                        const float4 pv = *reinterpret_cast<const float4*>(ps + row * C::GP + 4 * q4);
-                        pj[4 * q4 + 0] = pv.x;
-                        pj[4 * q4 + 1] = pv.y;
-                        pj[4 * q4 + 2] = pv.z;
-                        pj[4 * q4 + 3] = pv.w;
-                    }
-                    uint64_t v2[DPL / 2];
-                    const bool valid = row < cnt;
-#pragma unroll
-                    for (int i = 0; i < NCH; ++i) {
-                        uint4 w = *reinterpret_cast<const uint4*>(vt + row * kRowBytes + 16 * (sl + LPR * i));
-                        if (!valid) w = make_uint4(0u, 0u, 0u, 0u);  // stale bytes may not be finite
-                        v2[4 * i + 0] = bf2_to_f2(w.x);
-                        v2[4 * i + 1] = bf2_to_f2(w.y);
-                        v2[4 * i + 2] = bf2_to_f2(w.z);
-                        v2[4 * i + 3] = bf2_to_f2(w.w);
-                    }
-#pragma unroll
-                    for (int j = 0; j < G; ++j) {
-                        const uint64_t pp = pk(pj[j], pj[j]);
-#pragma unroll
-                        for (int i = 0; i < DPL / 2; ++i) o2[j][i] = fma2(pp, v2[i], o2[j][i]);
-                    }
+                cursor_next<TR>(cp, a, tab, hend, wA, wB);
+                if (++stage == NS) {
+                    stage = 0;
+                    phase ^= 1u;
                 }
             }
-            __syncwarp();
-            // Refill this stage with the tile NS ahead.
-            if (!dead && ld.h < hend) {
-                if (lane == 0) issue(ld, stage);
-                ++inflight;
-                cursor_next<TR, NW>(ld, a, tab, hend, A, Bc, warp);
-            }
-            cursor_next<TR, NW>(cp, a, tab, hend, A, Bc, warp);
-            if (++stage == NS) {
-                stage = 0;
-                phase ^= 1u;
+            if (dead) break;
+            finish_state<C>(S, l_all);
+            if (h == hlast) {
+                have_last = true;  // merged with the other warps at the end
+                if (lane == 0) seg_last[warp] = h;
+            } else if (h == hfirst) {
+                const int64_t rec = (int64_t)c * NW + warp;  // this slab continues in an earlier warp
+                store_state<C>(S, l_all, a.warp_o + rec * G * kHeadDim, a.warp_ml + rec * G * 2, lane);
+                if (lane == 0) seg_first[warp] = h;
+            } else if (FUSED) {
+                write_out_state<C>(a, S, l_all, b, g, lane);  // the whole slab lies in this warp's range
+            } else {
+                const int64_t slot = (int64_t)c + h;  // the whole slab lies in this warp's range
+                store_state<C>(S, l_all, a.work_o + slot * G * kHeadDim, a.work_ml + slot * G * 2, lane);
             }
         }
 
-        // Warp state of this segment: o summed over the RPS row lanes (same m), l
-        // summed over the TR lanes of each head, then broadcast per head.
-#pragma unroll
-        for (int o = LPR; o < 32; o <<= 1)
-#pragma unroll
-            for (int j = 0; j < G; ++j)
-#pragma unroll
-                for (int i = 0; i < DPL / 2; ++i) {
-                    const float2 f = upk(o2[j][i]);
-                    o2[j][i] = add2(o2[j][i], pk(__shfl_xor_sync(kFull, f.x, o), __shfl_xor_sync(kFull, f.y, o)));
+        if (dead) {
+            // After a timeout, wait (with the same bound) for the copies still in flight.
+            if (lane == 0)
+                for (int k = 0; k < inflight; ++k) {
+                    mbar_wait(smem_u32(&my_bars[stage]), phase);
+                    if (++stage == NS) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
                 }
-        float l_all[G];
-#pragma unroll
-        for (int u = 0; u < NSUM; ++u) {
-            float x = l_my[u];
-#pragma unroll
-            for (int o = TR / 2; o >= 1; o >>= 1) x += __shfl_xor_sync(kFull, x, o);
-            l_my[u] = x;
         }
-#pragma unroll
-        for (int j = 0; j < G; ++j) l_all[j] = __shfl_sync(kFull, l_my[(j * TR) / 32], (j * TR) % 32);
-
-        __syncthreads();  // every warp is done with its red/ps scratch, which mrg overlaps
-        float* mw = mrg + warp * G * (kHeadDim + 2);
-        if (r == 0) {
-#pragma unroll
-            for (int j = 0; j < G; ++j) {
-#pragma unroll
-                for (int i = 0; i < NCH; ++i) {
-                    // (kHeadDim + 2) floats per head is not 16-byte aligned: plain stores.
-                    float* d = mw + j * (kHeadDim + 2) + 8 * (sl + LPR * i);
-                    const float2 a0 = upk(o2[j][4 * i + 0]), a1 = upk(o2[j][4 * i + 1]);
-                    const float2 a2 = upk(o2[j][4 * i + 2]), a3 = upk(o2[j][4 * i + 3]);
-                    d[0] = a0.x; d[1] = a0.y; d[2] = a1.x; d[3] = a1.y;
-                    d[4] = a2.x; d[5] = a2.y; d[6] = a3.x; d[7] = a3.y;
-                }
-                if (sl == 0) {
-                    mw[j * (kHeadDim + 2) + kHeadDim] = m_all[j];
-                    mw[j * (kHeadDim + 2) + kHeadDim + 1] = l_all[j];
-                }
-            }
-        }
-        __syncthreads();
-        // Merge the NW warp states into the CTA's partial for slab h.
-        const int64_t slot = (int64_t)c + h;
-        for (int i = threadIdx.x; i < G * kHeadDim; i += NW * 32) {
-            const int j = i / kHeadDim, d = i - j * kHeadDim;
-            float M = -INFINITY;
-#pragma unroll
-            for (int w = 0; w < NW; ++w) M = fmaxf(M, mrg[(w * G + j) * (kHeadDim + 2) + kHeadDim]);
-            float O = 0.f, Lsum = 0.f;
-#pragma unroll
-            for (int w = 0; w < NW; ++w) {
-                const float* st = mrg + (w * G + j) * (kHeadDim + 2);
-                const float f = (st[kHeadDim] == -INFINITY) ? 0.f : ex2(st[kHeadDim] - M);
-                O = fmaf(st[d], f, O);
-                Lsum = fmaf(st[kHeadDim + 1], f, Lsum);
-            }
-            a.work_o[(slot * G + j) * kHeadDim + d] = O;
-            if (d == 0) {
-                a.work_ml[(slot * G + j) * 2] = M;
-                a.work_ml[(slot * G + j) * 2 + 1] = Lsum;
-            }
-        }
-        __syncthreads();  // mrg (and the warps' scratch) is reused by the next segment
     }
+    // The warp's own ring is idle now (every tile it issued was consumed): its
+    // final state goes there. Then the CTA merges, all warps sharing the work
+    // (one CTA per SM: warps that finish early have nothing else to run).
+    if (have_last)
+        store_state<C>(S, l_all, reinterpret_cast<float*>(my_ring), reinterpret_cast<float*>(my_ring) + G * kHeadDim,
+                       lane);
+    __syncthreads();
+    pdl_wait();  // the merges write the workspace and out: the previous kernel must be done with them
 
-    // After a timeout, wait (with the same bound) for the copies this warp still has in flight.
-    if (dead && lane == 0) {
-        for (int k = 0; k < dead_inflight; ++k) {
-            mbar_wait(smem_u32(&my_bars[dead_stage]), dead_phase);
-            if (++dead_stage == NS) {
-                dead_stage = 0;
-                dead_phase ^= 1u;
-            }
+    // Entry e (lane e) is the first (even e) or last (odd e) slab of warp e/2, -1 if
+    // none; entries list their slabs in non-decreasing order. Task t = (slab #t/G,
+    // head t%G) for the distinct slabs; warp w takes tasks w, w+NW, ...
+    static_assert(2 * NW <= 32, "one entry per lane");
+    const int h_e = (lane < 2 * NW) ? ((lane & 1) ? seg_last[lane >> 1] : seg_first[lane >> 1]) : -1;
+    int prev = -1;  // slab of the nearest valid entry before this one
+#pragma unroll
+    for (int f = 0; f < 2 * NW; ++f) {
+        const int hf = __shfl_sync(kFull, h_e, f);
+        if (f < lane && hf >= 0) prev = hf;
+    }
+    const unsigned fresh = __ballot_sync(kFull, h_e >= 0 && h_e != prev);
+    const int nslab = __popc(fresh);
+    int32_t* last_flag = seg_first;  // reused after the entries are read: 1 if this CTA merges slab #i
+    for (int t = warp; t < nslab * G; t += NW) {
+        const int si = t / G, j = t - si * G;
+        unsigned m = fresh;
+        for (int k = 0; k < si; ++k) m &= m - 1;
+        const int h = __shfl_sync(kFull, h_e, __ffs(m) - 1);
+        const unsigned same = __ballot_sync(kFull, h_e == h);
+        int c0h = 0, c1h = 0;
+        const int nct =
+            FUSED ? ctas_of_slab(slab_start(a, tab, h), slab_start(a, tab, h + 1), R, a.nctas, &c0h, &c1h) : 0;
+        float M = -INFINITY;
+#pragma unroll
+        for (int f = 0; f < 2 * NW; ++f) {
+            if (!((same >> f) & 1u)) continue;
+            const int w = f >> 1;
+            const float* ml = (f & 1) ? reinterpret_cast<const float*>(smem + w * NS * C::kStageBytes) + G * kHeadDim
+                                      : a.warp_ml + ((int64_t)c * NW + w) * G * 2;
+            M = fmaxf(M, ml[2 * j]);
         }
+        float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
+        float L = 0.f;
+#pragma unroll
+        for (int f = 0; f < 2 * NW; ++f) {
+            if (!((same >> f) & 1u)) continue;
+            const int w = f >> 1;
+            const float* ob = (f & 1) ? reinterpret_cast<const float*>(smem + w * NS * C::kStageBytes)
+                                      : a.warp_o + ((int64_t)c * NW + w) * G * kHeadDim;
+            const float* ml = (f & 1) ? ob + G * kHeadDim : a.warp_ml + ((int64_t)c * NW + w) * G * 2;
+            const float2 mlj = *reinterpret_cast<const float2*>(ml + 2 * j);
+            const float fct = (mlj.x == -INFINITY) ? 0.f : ex2(mlj.x - M);
+            L = fmaf(mlj.y, fct, L);
+            const float4 v = reinterpret_cast<const float4*>(ob + j * kHeadDim)[lane];
+            O.x = fmaf(v.x, fct, O.x);
+            O.y = fmaf(v.y, fct, O.y);
+            O.z = fmaf(v.z, fct, O.z);
+            O.w = fmaf(v.w, fct, O.w);
+        }
+        if (FUSED && nct == 1) {
+            write_out<G>(a, h / a.Hkv, h % a.Hkv, j, O, L, lane);  // the slab lies wholly in this CTA
+        } else {
+            const int64_t slot = (int64_t)c + h;
+            reinterpret_cast<float4*>(a.work_o + (slot * G + j) * kHeadDim)[lane] = O;
+            if (lane == 0) *reinterpret_cast<float2*>(a.work_ml + (slot * G + j) * 2) = make_float2(M, L);
+        }
+    }
+    if (!FUSED) return;
+    __syncthreads();  // this CTA's partials are written (and seg_first may be reused)
+
+    // Count this CTA in for every shared slab; the last CTA of a slab merges it.
+    if (warp == 0) {
+        int flag = 0, c0h = 0, c1h = 0, h = -1;
+        if (lane < nslab) {
+            unsigned m = fresh;
+            for (int k = 0; k < lane; ++k) m &= m - 1;
+            h = __ffs(m) - 1;  // entry index; slab below
+        }
+        const int hh = __shfl_sync(kFull, h_e, h < 0 ? 0 : h);
+        if (lane < nslab) {
+            const int nct = ctas_of_slab(slab_start(a, tab, hh), slab_start(a, tab, hh + 1), R, a.nctas, &c0h, &c1h);
+            if (nct > 1) {
+                __threadfence();
+                flag = (atomicAdd(&a.slab_count[hh], 1) == nct - 1) ? 1 : 0;
+                if (flag) {
+                    __threadfence();
+                    a.slab_count[hh] = 0;  // ready for the next call
+                }
+            }
+            last_flag[lane] = flag;
+        }
+    }
+    __syncthreads();
+    for (int t = warp; t < nslab * G; t += NW) {
+        const int si = t / G, j = t - si * G;
+        if (!last_flag[si]) continue;
+        unsigned m = fresh;
+        for (int k = 0; k < si; ++k) m &= m - 1;
+        const int h = __shfl_sync(kFull, h_e, __ffs(m) - 1);
+        int c0h = 0, c1h = 0;
+        ctas_of_slab(slab_start(a, tab, h), slab_start(a, tab, h + 1), R, a.nctas, &c0h, &c1h);
+        merge_slab_head<G>(a, h, j, c0h, c1h, R, lane);
     }
 }
 
 // ------------------------------------------------------------ combine kernel
-// One CTA per (b, q-head): kCombineWarps warps split the slab's partials,
-// each keeps its loads in flight, then the CTA sums the warps' shares.
-constexpr int kCombineWarps = 4;
+// One CTA per (b, q-head): the CTA's threads find the max over the slab's
+// partials, its warps split the partials (loads kept in flight), and the
+// CTA sums the warps' shares.
+constexpr int kCombineWarps = 8;
 constexpr int kCombineStride = kHeadDim + 4;  // floats per warp share: o[128], L, pad (16-byte rows)
 
 __global__ void __launch_bounds__(kCombineWarps * 32) decode_combine_kernel(const DecodeArgs a)
@@ -664,41 +911,52 @@ __global__ void __launch_bounds__(kCombineWarps * 32) decode_combine_kernel(cons
     SeqTable tab{csmem, csmem + a.B};
     // [kCombineWarps][kCombineStride] floats after the table, at a 16-byte boundary.
     float* red = reinterpret_cast<float*>(csmem + (((2 * a.B + 1) + 3) & ~3));
+    __shared__ float wmax[kCombineWarps];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    pdl_launch_dependents();
     if (warp == 0) build_seq_table(a, tab, false);
     __syncthreads();
+    pdl_wait();  // the partials of the previous (partial) kernel
 
     const int pair = blockIdx.x;  // (b, q-head)
     const int b = pair / a.H, hq = pair - b * a.H;
     const int g = hq / a.G, j = hq - g * a.G;
     const int h = b * a.Hkv + g;
     const int NHl = a.B * a.Hkv;
-    const int64_t R = slab_start(a, tab, NHl);
-    const int64_t p0 = slab_start(a, tab, h), p1 = slab_start(a, tab, h + 1);
+    const int R = slab_start(a, tab, NHl);
+    const int p0 = slab_start(a, tab, h), p1 = slab_start(a, tab, h + 1);
+    float4* outp = reinterpret_cast<float4*>(a.out + ((int64_t)b * a.H + hq) * kHeadDim);
+    if (p1 <= p0) {  // no rows: zeros (uniform over the CTA)
+        if (warp == 0) outp[lane] = make_float4(0.f, 0.f, 0.f, 0.f);
+        return;
+    }
+    const int P = a.nctas;
+    const int c0 = part_of(p0, R, P), c1 = part_of(p1 - 1, R, P);
+    float M = -INFINITY;
+    for (int c = c0 + (int)threadIdx.x; c <= c1; c += kCombineWarps * 32)
+        if (part_start(c, R, P) < part_start(c + 1, R, P))
+            M = fmaxf(M, a.work_ml[(((int64_t)c + h) * a.G + j) * 2]);
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) M = fmaxf(M, __shfl_xor_sync(kFull, M, o));
+    if (lane == 0) wmax[warp] = M;
+    __syncthreads();
+#pragma unroll
+    for (int w = 0; w < kCombineWarps; ++w) M = fmaxf(M, wmax[w]);
+
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
     float Lw = 0.f;
-    if (p1 > p0) {
-        const int c0 = cta_of(p0, R, a.nctas), c1 = cta_of(p1 - 1, R, a.nctas);
-        // Global max over the partials (lanes in parallel), same in every warp.
-        float M = -INFINITY;
-        for (int cc = c0 + lane; cc <= c1; cc += 32)
-            if (cta_start(cc, R, a.nctas) < cta_start(cc + 1, R, a.nctas))
-                M = fmaxf(M, a.work_ml[(((int64_t)cc + h) * a.G + j) * 2]);
-#pragma unroll
-        for (int o = 16; o >= 1; o >>= 1) M = fmaxf(M, __shfl_xor_sync(kFull, M, o));
 #pragma unroll 4
-        for (int cc = c0 + warp; cc <= c1; cc += kCombineWarps) {
-            if (cta_start(cc, R, a.nctas) == cta_start(cc + 1, R, a.nctas)) continue;
-            const int64_t sj = ((int64_t)cc + h) * a.G + j;
-            const float mc = a.work_ml[sj * 2], lc = a.work_ml[sj * 2 + 1];
-            const float f = (mc == -INFINITY) ? 0.f : ex2(mc - M);
-            Lw = fmaf(lc, f, Lw);
-            const float4 v = *reinterpret_cast<const float4*>(a.work_o + sj * kHeadDim + 4 * lane);
-            acc.x = fmaf(v.x, f, acc.x);
-            acc.y = fmaf(v.y, f, acc.y);
-            acc.z = fmaf(v.z, f, acc.z);
-            acc.w = fmaf(v.w, f, acc.w);
-        }
+    for (int c = c0 + warp; c <= c1; c += kCombineWarps) {
+        if (part_start(c, R, P) == part_start(c + 1, R, P)) continue;
+        const int64_t sj = ((int64_t)c + h) * a.G + j;
+        const float2 ml = *reinterpret_cast<const float2*>(a.work_ml + sj * 2);
+        const float f = (ml.x == -INFINITY) ? 0.f : ex2(ml.x - M);
+        Lw = fmaf(ml.y, f, Lw);
+        const float4 v = *reinterpret_cast<const float4*>(a.work_o + sj * kHeadDim + 4 * lane);
+        acc.x = fmaf(v.x, f, acc.x);
+        acc.y = fmaf(v.y, f, acc.y);
+        acc.z = fmaf(v.z, f, acc.z);
+        acc.w = fmaf(v.w, f, acc.w);
     }
     float* rw = red + warp * kCombineStride;
     reinterpret_cast<float4*>(rw)[lane] = acc;
@@ -717,11 +975,7 @@ __global__ void __launch_bounds__(kCombineWarps * 32) decode_combine_kernel(cons
             L += red[w * kCombineStride + kHeadDim];
         }
         const float inv = L > 0.f ? 1.f / L : 0.f;
-        o.x *= inv;
-        o.y *= inv;
-        o.z *= inv;
-        o.w *= inv;
-        *reinterpret_cast<float4*>(a.out + ((int64_t)b * a.H + hq) * kHeadDim + 4 * lane) = o;
+        outp[lane] = make_float4(o.x * inv, o.y * inv, o.z * inv, o.w * inv);
     }
 }
 
@@ -736,16 +990,40 @@ __global__ void advance_kernel(int32_t* n_app, int B, int reserve, int32_t* stat
 }
 
 // ------------------------------------------------------------ launch table
-// G <= 4: a quarter-warp per row (16 dims a lane), 16-row tiles, 3 stages.
-// G >= 5: a half-warp per row (8 dims a lane), 8-row tiles, 5 stages.
+// G <= 4: 8 lanes a row (16 dims each), 16-row tiles, 3 stages, 8 warps.
+// G >= 5: 16 lanes a row (8 dims each), 8-row tiles, 5 stages, 8 warps.
+#ifndef DKV_CFG_SMALL_G
+#define DKV_CFG_SMALL_G 8, 16, 3, 8
+#endif
+#ifndef DKV_CFG_LARGE_G
+#define DKV_CFG_LARGE_G 16, 8, 5, 8
+#endif
 template <int G>
-using PKFor = typename std::conditional<(G <= 4), PK<G, 8, 16, 3, 8>, PK<G, 16, 8, 5, 8>>::type;
+using PKFor = typename std::conditional<(G <= 4), PK<G, DKV_CFG_SMALL_G>, PK<G, DKV_CFG_LARGE_G>>::type;
 
-template <int G>
+// Launch with programmatic stream serialization: the kernel may start while the
+// previous kernel in the stream drains, and waits (griddepcontrol.wait) before
+// it reads that kernel's results.
+template <class K>
+cudaError_t launch_pdl(K kernel, int grid, int block, int smem, cudaStream_t st, const DecodeArgs& a)
+{
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = dim3(grid);
+    lc.blockDim = dim3(block);
+    lc.dynamicSmemBytes = smem;
+    lc.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    lc.attrs = attr;
+    lc.numAttrs = 1;
+    return cudaLaunchKernelEx(&lc, kernel, a);
+}
+
+template <int G, bool FUSED>
 cudaError_t launch_partial_g(const DecodeArgs& a, const DecodeConfig& cfg, cudaStream_t st)
 {
-    decode_partial_kernel<PKFor<G>><<<cfg.nctas, PKFor<G>::NW * 32, cfg.smem_bytes, st>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(decode_partial_kernel<PKFor<G>, FUSED>, cfg.nctas, PKFor<G>::NW * 32, cfg.smem_bytes, st, a);
 }
 
 template <int G>
@@ -753,16 +1031,28 @@ cudaError_t config_g(int B, DecodeConfig* cfg)
 {
     using C = PKFor<G>;
     const int smem = C::bytes(B);
-    cudaError_t e = cudaFuncSetAttribute(decode_partial_kernel<C>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaError_t e = cudaFuncSetAttribute(decode_partial_kernel<C, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         smem);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(decode_partial_kernel<C, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     int dev = 0, sms = 0, per_sm = 0;
     if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
     if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-    if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_partial_kernel<C>, C::NW * 32, smem)) !=
+    if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_partial_kernel<C, true>, C::NW * 32, smem)) !=
         cudaSuccess)
         return e;
     if (per_sm < 1) return cudaErrorInvalidConfiguration;
+    // The small kernels between partial launches ask for the same shared-memory
+    // carve-out, so the SMs need not reconfigure L1 between launches.
+    if ((e = cudaFuncSetAttribute(decode_combine_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                  cudaSharedmemCarveoutMaxShared)) != cudaSuccess)
+        return e;
+    if ((e = cudaFuncSetAttribute(advance_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                  cudaSharedmemCarveoutMaxShared)) != cudaSuccess)
+        return e;
     cfg->nctas = sms * per_sm;
+    cfg->nwarps = C::NW;
     cfg->smem_bytes = smem;
     return cudaSuccess;
 }
@@ -785,27 +1075,37 @@ cudaError_t decode_config(int G, int B, DecodeConfig* cfg)
     }
 }
 
-cudaError_t launch_decode_partial(const DecodeArgs& a, const DecodeConfig& cfg, cudaStream_t st)
+template <bool FUSED>
+cudaError_t launch_partial_any(const DecodeArgs& a, const DecodeConfig& cfg, cudaStream_t st)
 {
     switch (a.G) {
-        case 1: return launch_partial_g<1>(a, cfg, st);
-        case 2: return launch_partial_g<2>(a, cfg, st);
-        case 3: return launch_partial_g<3>(a, cfg, st);
-        case 4: return launch_partial_g<4>(a, cfg, st);
-        case 5: return launch_partial_g<5>(a, cfg, st);
-        case 6: return launch_partial_g<6>(a, cfg, st);
-        case 7: return launch_partial_g<7>(a, cfg, st);
-        case 8: return launch_partial_g<8>(a, cfg, st);
+        case 1: return launch_partial_g<1, FUSED>(a, cfg, st);
+        case 2: return launch_partial_g<2, FUSED>(a, cfg, st);
+        case 3: return launch_partial_g<3, FUSED>(a, cfg, st);
+        case 4: return launch_partial_g<4, FUSED>(a, cfg, st);
+        case 5: return launch_partial_g<5, FUSED>(a, cfg, st);
+        case 6: return launch_partial_g<6, FUSED>(a, cfg, st);
+        case 7: return launch_partial_g<7, FUSED>(a, cfg, st);
+        case 8: return launch_partial_g<8, FUSED>(a, cfg, st);
         default: return cudaErrorInvalidValue;
     }
+}
+
+cudaError_t launch_decode_partial(const DecodeArgs& a, const DecodeConfig& cfg, cudaStream_t st)
+{
+    return launch_partial_any<false>(a, cfg, st);
+}
+
+cudaError_t launch_decode_fused(const DecodeArgs& a, const DecodeConfig& cfg, cudaStream_t st)
+{
+    return launch_partial_any<true>(a, cfg, st);
 }
 
 cudaError_t launch_decode_combine(const DecodeArgs& a, cudaStream_t st)
 {
     const int pairs = a.B * a.H;
     const int smem = (2 * a.B + 1) * 4 + 16 + kCombineWarps * kCombineStride * 4;
-    decode_combine_kernel<<<pairs, kCombineWarps * 32, smem, st>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(decode_combine_kernel, pairs, kCombineWarps * 32, smem, st, a);
 }
 
 cudaError_t launch_advance(int32_t* n_app, int B, int reserve, int32_t* status, cudaStream_t st)

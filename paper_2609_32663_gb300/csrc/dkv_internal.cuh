@@ -57,30 +57,40 @@ struct DecodeArgs {
     const int32_t* len;     // layer slice [NHl]
     const int64_t* off;     // layer slice [NHl]
     const int64_t* ioff;    // layer slice [NHl+1] (absolute; the layer prefix is ioff[h]-ioff[0])
-    float* work_o;          // [slots][G][128]
+    float* work_o;          // [slots][G][128], one slot per (CTA, slab) partial
     float* work_ml;         // [slots][G][2]
+    float* warp_o;          // [nparts][G][128]: a warp's state for a slab it left mid-range
+    float* warp_ml;         // [nparts][G][2]
     float* out;             // [B][H][128]
+    int32_t* slab_count;    // [B*Hkv] arrival counters of the fused merge (zero between calls)
     int32_t* status;
     int B, H, Hkv, G;
     int reserve;
     int append;             // 1 when k_new/v_new are given
     float qscale;           // softmax scale * log2(e)
-    int nctas;              // CTAs of the split-K grid (the partition's P)
+    int nctas;              // CTAs of the split-K grid: the row partition's part count
 };
-
-// Slots of split-K partials a decode call can write: nctas + heads per layer.
-inline int64_t decode_slots(int nctas, int heads_per_layer) {
-    return (int64_t)nctas + heads_per_layer;
-}
 
 struct DecodeConfig {
     int nctas;        // grid of the partial kernel
+    int nwarps;       // warps per CTA of the partial kernel
     int smem_bytes;   // dynamic shared memory of the partial kernel
 };
+
+// Floats of split-K workspace a decode call needs for group size G: one
+// (o[128], m, l) record per head of the group for every (CTA, slab) slot
+// (nctas + slabs per layer) and for every warp of the grid.
+inline int64_t decode_workspace_floats(const DecodeConfig& c, int G, int heads_per_layer) {
+    const int64_t records = (int64_t)c.nctas + heads_per_layer + (int64_t)c.nctas * c.nwarps;
+    return records * G * (128 + 2);
+}
 // Grid and shared memory of the partial kernel for group size G on this device.
 cudaError_t decode_config(int G, int B, DecodeConfig* cfg);
 // Split-K partials of one layer into the workspace, then the per-(b, q-head) merge.
 cudaError_t launch_decode_partial(const DecodeArgs& a, const DecodeConfig& cfg, cudaStream_t st);
+// The partial pass with the combine fused in: the last CTA to finish a slab merges
+// the slab's partials and writes out (uses a.slab_count).
+cudaError_t launch_decode_fused(const DecodeArgs& a, const DecodeConfig& cfg, cudaStream_t st);
 cudaError_t launch_decode_combine(const DecodeArgs& a, cudaStream_t st);
 cudaError_t launch_advance(int32_t* n_app, int B, int reserve, int32_t* status, cudaStream_t st);
 

@@ -23,8 +23,8 @@
 
 namespace {
 
-// 8 MiB: partials of up to (CTAs + sequences x KV heads) slots x group size x
-// 130 floats, plus one status word at the end.
+// 8 MiB: split-K records of (CTAs + sequences x KV heads + warps of the grid) x
+// group size x 130 floats, plus one status word at the end.
 constexpr size_t kScratchBytes = size_t(8) << 20;
 constexpr size_t kStatusOffset = kScratchBytes - 256;
 
@@ -99,8 +99,8 @@ extern "C" dkv_status dkv_decode_attn_noalloc(const dkv_shape* s, int32_t B, int
     if ((e = dkv::decode_config(G, B, &cfg)) != cudaSuccess)
         return bad(DKV_ERR_CUDA, "decode_config: %s", cudaGetErrorString(e));
     const int NHl = B * s->H_kv;
-    const int64_t slots = dkv::decode_slots(cfg.nctas, NHl);
-    const size_t need = (size_t)slots * G * (dkv::kHeadDim + 2) * sizeof(float);
+    const int64_t slots = (int64_t)cfg.nctas + NHl;
+    const size_t need = (size_t)dkv::decode_workspace_floats(cfg, G, NHl) * sizeof(float);
     if (need > kStatusOffset)
         return bad(DKV_ERR_INVALID_ARG,
                    "split-K partials need %zu bytes (%lld slots x G=%d); the static scratch holds %zu", need,
@@ -125,7 +125,9 @@ extern "C" dkv_status dkv_decode_attn_noalloc(const dkv_shape* s, int32_t B, int
     a.off = d_off + (int64_t)layer * NHl;
     a.ioff = d_ioff + (int64_t)layer * NHl;
     a.work_o = work;
-    a.work_ml = work + (size_t)slots * G * dkv::kHeadDim;
+    a.work_ml = a.work_o + (size_t)slots * G * dkv::kHeadDim;
+    a.warp_o = a.work_ml + (size_t)slots * G * 2;
+    a.warp_ml = a.warp_o + (size_t)cfg.nctas * cfg.nwarps * G * dkv::kHeadDim;
     a.out = out;
     a.status = status_word;
     a.B = B;

@@ -139,6 +139,46 @@ def test_decode_outlier_keys_and_custom_scale():
     c.close()
 
 
+@pytest.mark.parametrize("G", [4, 7])
+def test_separate_partial_and_combine_entry_points(G):
+    """dkv_decode_partial + dkv_decode_combine (two launches) give the oracle's answer,
+    with this step's token appended, like dkv_decode_attn does in one launch."""
+    w = wl(H=2 * G, Hkv=2, T=7000, B=3, D=8, W=800, ragged=(500, 7000), seed=40 + G)
+    c = Case(w, reserve=3)
+    q, kn, vn = I.decode_inputs(w, 2)
+    n_app = torch.zeros(w.B, dtype=torch.int32, device=c.dev)
+    na = np.zeros(w.B, np.int32)
+    out = torch.full((w.B, w.H, 128), float("nan"), dtype=torch.float32, device=c.dev)
+    for s in range(2):
+        for layer in range(w.L):
+            dkv.dkv_decode_partial(c.plan, layer, q[s, layer].to(c.dev), kn[s, layer].to(c.dev),
+                                   vn[s, layer].to(c.dev), n_app, c.Kc, c.Vc)
+            dkv.dkv_decode_combine(c.plan, layer, n_app, True, out)
+            O.append(c.om, layer, w.B, w.Hkv, c.reserve, na, I.bf16_bits(kn[s, layer]), I.bf16_bits(vn[s, layer]),
+                     c.oKc, c.oVc)
+            want = O.decode(c.om, layer, w.B, w.H, w.Hkv, I.bf16_bits(q[s, layer]), c.oKc, c.oVc, n_rows_app=na + 1)
+            assert_close(out.cpu().numpy(), want, f"two-launch step {s} layer {layer}")
+        dkv.dkv_advance(c.plan, n_app)
+        na += 1
+    c.check_packed_with_appends(na)
+    c.close()
+
+
+def test_decode_repeated_calls_reuse_counters():
+    """Many consecutive single-launch calls on one plan (the fused combine's slab
+    counters reset themselves) stay equal to the oracle."""
+    w = wl(H=8, Hkv=2, T=9000, B=2, D=8, W=(9000 - 1152) // 8 + 1, ragged=(2000, 9000), seed=51)
+    c = Case(w)
+    q, _, _ = I.decode_inputs(w, 1)
+    out = torch.empty((w.B, w.H, 128), dtype=torch.float32, device=c.dev)
+    want = [O.decode(c.om, l, w.B, w.H, w.Hkv, I.bf16_bits(q[0, l]), c.oKc, c.oVc) for l in range(w.L)]
+    for rep in range(6):
+        for layer in range(w.L):
+            dkv.dkv_decode_attn(c.plan, layer, q[0, layer].to(c.dev), None, None, None, c.Kc, c.Vc, out)
+            assert_close(out.cpu().numpy(), want[layer], f"rep {rep} layer {layer}")
+    c.close()
+
+
 def test_all_keep_equals_dense_plan():
     """M = 1 gives the same output as the dense-cache plan over the uncompressed K/V."""
     w = wl(H=8, Hkv=2, T=7000, B=2, D=8, W=800, ragged=(3000, 7000), seed=9)
