@@ -229,8 +229,7 @@ dkv_status dkv_plan_status(const dkv_plan* plan, int32_t* word, int32_t clear, c
  *
  * The split-K partials live in a fixed 8 MiB array inside the library image,
  * held on every GPU that loads the library until the process exits; a call
- * whose split-K records ((17 x SM count + B*H_kv) x G x 130 floats for G <= 4,
- * (9 x SM count + B*H_kv) x G x 130 for G > 4) do not fit gets
+ * whose split-K records ((9 x SM count + B*H_kv) x G x 130 floats) do not fit gets
  * DKV_ERR_INVALID_ARG. The first call on each device looks up that array's
  * device address (a one-time set-up per device); make that first call before
  * any stream capture. Every call reuses the same array, so calls whose kernels

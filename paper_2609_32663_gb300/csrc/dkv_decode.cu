@@ -33,6 +33,7 @@ constexpr unsigned kFull = 0xffffffffu;
 constexpr int kMaxB = 512;
 constexpr int kWaitSpins = 1 << 22;  // bound on mbarrier polls (each poll may suspend)
 constexpr float kSlack = 8.f;        // lazy-rescale threshold of the online softmax (log2 units)
+constexpr int PRE = 1;               // tiles a warp fetches before waiting for the previous kernel
 
 // ------------------------------------------------------------ PTX helpers
 __device__ __forceinline__ uint32_t smem_u32(const void* p)
@@ -682,12 +683,12 @@ __global__ void __launch_bounds__(C::NW * 32, 1) decode_partial_kernel(const Dec
         int inflight = 0;
         if (lane == 0) {
             Cursor it = ld;
-            for (int s = 0; s < NS && it.h < hend; ++s) {
+            for (int s = 0; s < PRE && it.h < hend; ++s) {
                 issue(it, s);
                 cursor_next<TR>(it, a, tab, hend, wA, wB);
             }
         }
-        for (int s = 0; s < NS && ld.h < hend; ++s) {
+        for (int s = 0; s < PRE && ld.h < hend; ++s) {
             ++inflight;
             cursor_next<TR>(ld, a, tab, hend, wA, wB);
         }
@@ -695,6 +696,17 @@ __global__ void __launch_bounds__(C::NW * 32, 1) decode_partial_kernel(const Dec
         // earlier steps; q, k_new, v_new, the cache slots written here and the
         // workspace belong to the previous kernel's epoch.
         pdl_wait();
+        if (lane == 0) {
+            Cursor it = ld;
+            for (int s = PRE; s < NS && it.h < hend; ++s) {
+                issue(it, s);
+                cursor_next<TR>(it, a, tab, hend, wA, wB);
+            }
+        }
+        for (int s = PRE; s < NS && ld.h < hend; ++s) {
+            ++inflight;
+            cursor_next<TR>(ld, a, tab, hend, wA, wB);
+        }
         int stage = 0;
         uint32_t phase = 0;
         const float cs = a.qscale;  // softmax scale * log2(e)
@@ -875,12 +887,10 @@ __global__ void __launch_bounds__(C::NW * 32, 1) decode_partial_kernel(const Dec
         if (lane < nslab) {
             const int nct = ctas_of_slab(slab_start(a, tab, hh), slab_start(a, tab, hh + 1), R, a.nctas, &c0h, &c1h);
             if (nct > 1) {
-                __threadfence();
-                flag = (atomicAdd(&a.slab_count[hh], 1) == nct - 1) ? 1 : 0;
-                if (flag) {
-                    __threadfence();
-                    a.slab_count[hh] = 0;  // ready for the next call
-                }
+                int old;
+                asm volatile("atom.add.acq_rel.gpu.s32 %0, [%1], 1;" : "=r"(old) : "l"(&a.slab_count[hh]) : "memory");
+                flag = (old == nct - 1) ? 1 : 0;
+                if (flag) a.slab_count[hh] = 0;  // ready for the next call
             }
             last_flag[lane] = flag;
         }
