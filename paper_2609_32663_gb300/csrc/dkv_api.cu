@@ -29,7 +29,7 @@ struct dkv_plan {
     int32_t* d_idx = nullptr;   // [kept]
     int32_t* d_status = nullptr;
     float* d_work = nullptr;    // split-K partials
-    int32_t* d_slab_count = nullptr;  // [B*H_kv] arrival counters of the fused combine
+    int32_t* d_slab_count = nullptr;  // [B*H_kv][G] arrival counters of the fused combine
     dkv::DecodeConfig cfg{};
     int64_t slots = 0;
 };
@@ -135,9 +135,9 @@ dkv_status finish_plan(dkv_plan* p)
     st = dalloc(&p->d_status, 1, "status word");
     if (st != DKV_OK) return st;
     if ((e = cudaMemset(p->d_status, 0, sizeof(int32_t))) != cudaSuccess) return cuda_fail(e, "cudaMemset");
-    st = dalloc(&p->d_slab_count, (size_t)p->B * p->s.H_kv, "slab counters");
+    st = dalloc(&p->d_slab_count, (size_t)p->B * p->s.H_kv * p->G, "slab counters");
     if (st != DKV_OK) return st;
-    if ((e = cudaMemset(p->d_slab_count, 0, sizeof(int32_t) * p->B * p->s.H_kv)) != cudaSuccess)
+    if ((e = cudaMemset(p->d_slab_count, 0, sizeof(int32_t) * p->B * p->s.H_kv * p->G)) != cudaSuccess)
         return cuda_fail(e, "cudaMemset");
     return DKV_OK;
 }

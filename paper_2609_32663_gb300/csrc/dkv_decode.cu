@@ -164,7 +164,7 @@ __device__ __forceinline__ int part_start(int w, int R, int P)
 // Largest part w with part_start(w) <= x, for 0 <= x < R.
 __device__ __forceinline__ int part_of(int x, int R, int P)
 {
-    int w = (int)(((int64_t)x * P) / R);
+    int w = min(P - 1, (int)((float)x * ((float)P / (float)R)));  // estimate, then exact steps
     while (w + 1 < P && part_start(w + 1, R, P) <= x) ++w;
     while (w > 0 && part_start(w, R, P) > x) --w;
     return w;
@@ -475,53 +475,46 @@ __device__ __forceinline__ void write_out(const DecodeArgs& a, int b, int g, int
 template <int G>
 __device__ void merge_slab_head(const DecodeArgs& a, int h, int j, int c0, int c1, int R, int lane)
 {
+    // Every lane loads the (m, l) and its 4 dims of o of KB partials at once (one
+    // L2 round per batch), then merges them in registers; batches chain online.
+    constexpr int KB = 16;
     const int b = h / a.Hkv, g = h - b * a.Hkv;
-    const int n = c1 - c0 + 1;
     const int P = a.nctas;
     const bool all_live = R >= P;  // every CTA has rows
-    auto live = [&](int cc) { return all_live || part_start(cc, R, P) < part_start(cc + 1, R, P); };
-    float M = -INFINITY;
-    for (int base = 0; base < n; base += 32) {
-        const int cc = c0 + base + lane;
-        if (base + lane < n && live(cc)) M = fmaxf(M, __ldcg(a.work_ml + (((int64_t)cc + h) * G + j) * 2));
-    }
-#pragma unroll
-    for (int o = 16; o >= 1; o >>= 1) M = fmaxf(M, __shfl_xor_sync(kFull, M, o));
-    float L = 0.f;
+    float M = -INFINITY, L = 0.f;
     float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int base = 0; base < n; base += 32) {
-        const int cc = c0 + base + lane;
-        float f = 0.f;
-        if (base + lane < n && live(cc)) {
-            const float2 ml = __ldcg(reinterpret_cast<const float2*>(a.work_ml + (((int64_t)cc + h) * G + j) * 2));
-            f = (ml.x == -INFINITY) ? 0.f : ex2(ml.x - M);
-            L = fmaf(f, ml.y, L);
+    for (int k0 = c0; k0 <= c1; k0 += KB) {
+        float2 ml[KB];
+        float4 v[KB];
+#pragma unroll
+        for (int u = 0; u < KB; ++u) {
+            const int cc = k0 + u;
+            const bool ok = cc <= c1 && (all_live || part_start(cc, R, P) < part_start(cc + 1, R, P));
+            const int64_t sj = ((int64_t)cc + h) * G + j;
+            ml[u] = ok ? __ldcg(reinterpret_cast<const float2*>(a.work_ml + sj * 2)) : make_float2(-INFINITY, 0.f);
+            v[u] = ok ? __ldcg(reinterpret_cast<const float4*>(a.work_o + sj * kHeadDim) + lane)
+                      : make_float4(0.f, 0.f, 0.f, 0.f);
         }
-        const int cnt = min(32, n - base);
-        for (int k0 = 0; k0 < cnt; k0 += 4) {
-            float fk[4];
-            float4 v[4];
+        float Mb = M;
 #pragma unroll
-            for (int u = 0; u < 4; ++u) fk[u] = __shfl_sync(kFull, f, (k0 + u) & 31);
+        for (int u = 0; u < KB; ++u) Mb = fmaxf(Mb, ml[u].x);
+        const float fo = (M == -INFINITY) ? 0.f : ex2(M - Mb);
+        L *= fo;
+        O.x *= fo;
+        O.y *= fo;
+        O.z *= fo;
+        O.w *= fo;
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int ck = c0 + base + k0 + u;
-                v[u] = (k0 + u < cnt && live(ck))
-                           ? __ldcg(reinterpret_cast<const float4*>(a.work_o + (((int64_t)ck + h) * G + j) * kHeadDim) + lane)
-                           : make_float4(0.f, 0.f, 0.f, 0.f);
-            }
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const float w = (k0 + u < cnt) ? fk[u] : 0.f;
-                O.x = fmaf(w, v[u].x, O.x);
-                O.y = fmaf(w, v[u].y, O.y);
-                O.z = fmaf(w, v[u].z, O.z);
-                O.w = fmaf(w, v[u].w, O.w);
-            }
+        for (int u = 0; u < KB; ++u) {
+            const float f = (ml[u].x == -INFINITY) ? 0.f : ex2(ml[u].x - Mb);
+            L = fmaf(f, ml[u].y, L);
+            O.x = fmaf(f, v[u].x, O.x);
+            O.y = fmaf(f, v[u].y, O.y);
+            O.z = fmaf(f, v[u].z, O.z);
+            O.w = fmaf(f, v[u].w, O.w);
         }
+        M = Mb;
     }
-#pragma unroll
-    for (int o = 16; o >= 1; o >>= 1) L += __shfl_xor_sync(kFull, L, o);
     write_out<G>(a, b, g, j, O, L, lane);
 }
 
@@ -827,7 +820,6 @@ __global__ void __launch_bounds__(C::NW * 32, 1) decode_partial_kernel(const Dec
     }
     const unsigned fresh = __ballot_sync(kFull, h_e >= 0 && h_e != prev);
     const int nslab = __popc(fresh);
-    int32_t* last_flag = seg_first;  // reused after the entries are read: 1 if this CTA merges slab #i
     for (int t = warp; t < nslab * G; t += NW) {
         const int si = t / G, j = t - si * G;
         unsigned m = fresh;
@@ -866,45 +858,26 @@ __global__ void __launch_bounds__(C::NW * 32, 1) decode_partial_kernel(const Dec
         }
         if (FUSED && nct == 1) {
             write_out<G>(a, h / a.Hkv, h % a.Hkv, j, O, L, lane);  // the slab lies wholly in this CTA
-        } else {
-            const int64_t slot = (int64_t)c + h;
-            reinterpret_cast<float4*>(a.work_o + (slot * G + j) * kHeadDim)[lane] = O;
-            if (lane == 0) *reinterpret_cast<float2*>(a.work_ml + (slot * G + j) * 2) = make_float2(M, L);
+            continue;
         }
-    }
-    if (!FUSED) return;
-    __syncthreads();  // this CTA's partials are written (and seg_first may be reused)
-
-    // Count this CTA in for every shared slab; the last CTA of a slab merges it.
-    if (warp == 0) {
-        int flag = 0, c0h = 0, c1h = 0, h = -1;
-        if (lane < nslab) {
-            unsigned m = fresh;
-            for (int k = 0; k < lane; ++k) m &= m - 1;
-            h = __ffs(m) - 1;  // entry index; slab below
+        const int64_t slot = (int64_t)c + h;
+        reinterpret_cast<float4*>(a.work_o + (slot * G + j) * kHeadDim)[lane] = O;
+        if (lane == 0) *reinterpret_cast<float2*>(a.work_ml + (slot * G + j) * 2) = make_float2(M, L);
+        if (!FUSED) continue;
+        // Count this CTA in for (slab, head): release of the partial just written,
+        // and, for the last CTA, acquire of the others' before merging them.
+        __syncwarp();
+        int last = 0;
+        if (lane == 0) {
+            int32_t* ctr = a.slab_count + (int64_t)h * G + j;
+            int old;
+            asm volatile("atom.add.acq_rel.gpu.s32 %0, [%1], 1;" : "=r"(old) : "l"(ctr) : "memory");
+            last = (old == nct - 1) ? 1 : 0;
+            if (last) *ctr = 0;  // ready for the next call
         }
-        const int hh = __shfl_sync(kFull, h_e, h < 0 ? 0 : h);
-        if (lane < nslab) {
-            const int nct = ctas_of_slab(slab_start(a, tab, hh), slab_start(a, tab, hh + 1), R, a.nctas, &c0h, &c1h);
-            if (nct > 1) {
-                int old;
-                asm volatile("atom.add.acq_rel.gpu.s32 %0, [%1], 1;" : "=r"(old) : "l"(&a.slab_count[hh]) : "memory");
-                flag = (old == nct - 1) ? 1 : 0;
-                if (flag) a.slab_count[hh] = 0;  // ready for the next call
-            }
-            last_flag[lane] = flag;
-        }
-    }
-    __syncthreads();
-    for (int t = warp; t < nslab * G; t += NW) {
-        const int si = t / G, j = t - si * G;
-        if (!last_flag[si]) continue;
-        unsigned m = fresh;
-        for (int k = 0; k < si; ++k) m &= m - 1;
-        const int h = __shfl_sync(kFull, h_e, __ffs(m) - 1);
-        int c0h = 0, c1h = 0;
-        ctas_of_slab(slab_start(a, tab, h), slab_start(a, tab, h + 1), R, a.nctas, &c0h, &c1h);
-        merge_slab_head<G>(a, h, j, c0h, c1h, R, lane);
+        last = __shfl_sync(kFull, last, 0);
+        __syncwarp();
+        if (last) merge_slab_head<G>(a, h, j, c0h, c1h, R, lane);
     }
 }
 

@@ -62,7 +62,7 @@ struct DecodeArgs {
     float* warp_o;          // [nparts][G][128]: a warp's state for a slab it left mid-range
     float* warp_ml;         // [nparts][G][2]
     float* out;             // [B][H][128]
-    int32_t* slab_count;    // [B*Hkv] arrival counters of the fused merge (zero between calls)
+    int32_t* slab_count;    // [B*Hkv][G] arrival counters of the fused merge (zero between calls)
     int32_t* status;
     int B, H, Hkv, G;
     int reserve;
