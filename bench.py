@@ -34,6 +34,33 @@ sys.path.insert(0, ROOT)
 
 from paper_2609_32663_gb300 import inputs as I  # noqa: E402
 
+# DRAM traffic of the decode kernel from one ncu capture: dram__bytes_read.sum +
+# dram__bytes_write.sum of layer 0 of llama8b-128k-l4 (the per-layer sizes of
+# llama8b-128k, 4 layers), against that launch's algorithmic bytes. Traffic grows
+# with the rows a launch streams, so a launch of the full workload is credited
+# ratio x its own algorithmic bytes -- only while the kernel sources still hash to
+# the value the capture was taken on (else the traffic is unknown: null).
+DECODE_TRAFFIC = {
+    "sources": ("paper_2609_32663_gb300/csrc/dkv_decode.cu", "paper_2609_32663_gb300/csrc/dkv_internal.cuh"),
+    "sha256": "c18acecf8a7c5285f05173627fd31b0dfb60abd95d134a620be660c42e48edc8",
+    "dram_bytes": 192_968_448 + 2_764_288,
+    "algorithmic_bytes": 376_646 * 512 + 32 * 128 * (2 + 4),
+    "capture": "profiles/decode_partial_llama8b-128k-l4.md",
+}
+
+
+def decode_traffic_per_launch(bytes_per_launch):
+    """ncu-measured DRAM bytes of one decode launch scaled to `bytes_per_launch`, or None."""
+    import hashlib
+    h = hashlib.sha256()
+    for f in DECODE_TRAFFIC["sources"]:
+        with open(os.path.join(ROOT, f), "rb") as fh:
+            h.update(fh.read())
+    if h.hexdigest() != DECODE_TRAFFIC["sha256"]:
+        return None
+    return int(round(bytes_per_launch * DECODE_TRAFFIC["dram_bytes"] / DECODE_TRAFFIC["algorithmic_bytes"]))
+
+
 METRIC = "compacted decode-attention us/step (Llama-3.1-8B KV shape, 131072 ctx, 34.6% retention)"
 UNIT = "us/step"
 
@@ -438,7 +465,10 @@ def run_dkv(args, dist):
                      "launches_timed": steps * wl.L,
                      "how": "CUDA events around the timed graph replays; avg launch = region / (steps x layers)",
                      "isolated_launch_us": round(t_part * 1e6, 2), "isolated_launches": n_launch,
-                     "traffic": None},
+                     "traffic": decode_traffic_per_launch(part_bytes),
+                     "traffic_how": "ncu dram__bytes_read.sum + dram__bytes_write.sum of one launch of the "
+                                    "4-layer case with the same per-layer sizes, scaled by algorithmic bytes; "
+                                    "null if the kernel sources changed since"},
         "compaction": {"gbs": round(comp["gbs"], 1), "ms": round(comp["ms"], 3),
                        "frac_of_hbm": round(comp["gbs"] / peak, 4), "kept_rows": info.kept_rows},
         "map_ms": round(env["map_ms"], 2),
