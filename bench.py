@@ -86,22 +86,31 @@ class Dist:
         self.rank = int(os.environ.get("RANK", "0"))
         self.local = int(os.environ.get("LOCAL_RANK", "0"))
         self.pg = None
+        self.cuda = False
         if self.world > 1:
             import torch
             import torch.distributed as dist
-            backend = "nccl" if torch.cuda.is_available() else "gloo"
-            dist.init_process_group(backend)
+            self.cuda = torch.cuda.is_available()
+            if self.cuda:
+                # One GPU per rank: the rank's device is current before NCCL binds to it.
+                torch.cuda.set_device(self.local)
+                dist.init_process_group("nccl", device_id=torch.device("cuda", self.local))
+            else:
+                dist.init_process_group("gloo")
             self.pg = dist
 
     def barrier(self):
         if self.pg:
-            self.pg.barrier()
+            if self.cuda:
+                self.pg.barrier(device_ids=[self.local])
+            else:
+                self.pg.barrier()
 
     def max(self, x):
         if not self.pg:
             return x
         import torch
-        dev = "cuda" if torch.cuda.is_available() else "cpu"
+        dev = torch.device("cuda", self.local) if self.cuda else "cpu"
         t = torch.tensor([float(x)], dtype=torch.float64, device=dev)
         self.pg.all_reduce(t, op=self.pg.ReduceOp.MAX)
         return float(t.item())

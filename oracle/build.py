@@ -15,7 +15,7 @@ def build(force: bool = False) -> str:
     if not force and os.path.exists(LIB) and os.path.getmtime(LIB) >= os.path.getmtime(SRC):
         return LIB
     cc = os.environ.get("CC", "gcc")
-    tmp = LIB + ".tmp"
+    tmp = f"{LIB}.{os.getpid()}.tmp"  # concurrent builders never share a temporary
     subprocess.check_call([cc, "-O2", "-std=c11", "-fPIC", "-shared", "-Wall", "-Wextra",
                            "-o", tmp, SRC, "-lm"])
     os.replace(tmp, LIB)

@@ -4,6 +4,7 @@ Each .cu file compiles in its own nvcc process (in parallel), then nvcc links a
 shared library with the CUDA runtime linked statically. Only one -gencode:
 compute_103a -> sm_103a (GB300).
 """
+import fcntl
 import glob
 import os
 import subprocess
@@ -42,10 +43,25 @@ def up_to_date():
 
 
 def build_library(force=False, verbose=False, extra_flags=()):
-    """Compile every csrc/*.cu and link libdkv.so. Returns the library path."""
+    """Compile every csrc/*.cu and link libdkv.so. Returns the library path.
+
+    Processes that build at the same time (one per rank under torchrun, or test
+    workers) serialise on a lock file; the ones that wait find the library up to
+    date and return it."""
     if not force and up_to_date():
         return LIB
     os.makedirs(OBJDIR, exist_ok=True)
+    with open(os.path.join(OBJDIR, ".lock"), "w") as lock:
+        fcntl.flock(lock, fcntl.LOCK_EX)
+        try:
+            if not force and up_to_date():
+                return LIB
+            return _build_locked(verbose, extra_flags)
+        finally:
+            fcntl.flock(lock, fcntl.LOCK_UN)
+
+
+def _build_locked(verbose, extra_flags):
     nvcc = _nvcc()
 
     def compile_one(src):
