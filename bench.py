@@ -41,11 +41,12 @@ from paper_2609_32663_gb300 import inputs as I  # noqa: E402
 # ratio x its own algorithmic bytes -- only while the kernel sources still hash to
 # the value the capture was taken on (else the traffic is unknown: null).
 DECODE_TRAFFIC = {
-    "sources": ("paper_2609_32663_gb300/csrc/dkv_decode.cu", "paper_2609_32663_gb300/csrc/dkv_internal.cuh"),
-    "sha256": "c18acecf8a7c5285f05173627fd31b0dfb60abd95d134a620be660c42e48edc8",
-    "dram_bytes": 192_968_448 + 2_764_288,
-    "algorithmic_bytes": 376_646 * 512 + 32 * 128 * (2 + 4),
-    "capture": "profiles/decode_partial_llama8b-128k-l4.md",
+    "sources": ("paper_2609_32663_gb300/csrc/dkv_decode_mma.cu", "paper_2609_32663_gb300/csrc/dkv_decode_common.cuh",
+                "paper_2609_32663_gb300/csrc/dkv_internal.cuh"),
+    "sha256": None,  # no capture of this kernel version yet
+    "dram_bytes": None,
+    "algorithmic_bytes": None,
+    "capture": "profiles/decode_mma_llama8b-128k-l4.md",
 }
 
 
@@ -56,7 +57,7 @@ def decode_traffic_per_launch(bytes_per_launch):
     for f in DECODE_TRAFFIC["sources"]:
         with open(os.path.join(ROOT, f), "rb") as fh:
             h.update(fh.read())
-    if h.hexdigest() != DECODE_TRAFFIC["sha256"]:
+    if DECODE_TRAFFIC["sha256"] is None or h.hexdigest() != DECODE_TRAFFIC["sha256"]:
         return None
     return int(round(bytes_per_launch * DECODE_TRAFFIC["dram_bytes"] / DECODE_TRAFFIC["algorithmic_bytes"]))
 
@@ -65,11 +66,22 @@ METRIC = "compacted decode-attention us/step (Llama-3.1-8B KV shape, 131072 ctx,
 UNIT = "us/step"
 
 
+DEFAULT_STEPS = 256
+DEFAULT_WARMUP = 8
+
+
+def reserve_rows(steps, warmup):
+    """Rows each slab keeps free for appended tokens: every step the run makes
+    (the timed and warm-up graph replays, the instrumented eager steps, the e2e
+    run) appends one, with room to spare."""
+    return steps + warmup + 64
+
+
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=256)
-    ap.add_argument("--warmup", type=int, default=8)
+    ap.add_argument("--steps", type=int, default=DEFAULT_STEPS)
+    ap.add_argument("--warmup", type=int, default=DEFAULT_WARMUP)
     ap.add_argument("--impl", default="dkv", choices=["dkv", "reference"])
     ap.add_argument("--workload", default="llama8b-128k", choices=sorted(I.WORKLOADS))
     ap.add_argument("--no-dense", action="store_true", help="skip the dense-cache baseline")
@@ -416,7 +428,7 @@ def run_dkv(args, dist):
     steps, warmup = args.steps, max(args.warmup, 3)
     if args.profile:
         steps, warmup = min(steps, 2), min(warmup, 3)
-    reserve = steps + warmup + 64
+    reserve = reserve_rows(steps, warmup)
     env = setup(wl, dev, reserve)
     comp = time_compaction(env, reps=3 if args.profile else 10)
     info = env["info"]
@@ -467,7 +479,7 @@ def run_dkv(args, dist):
         "algorithmic_gb_per_step": round(algo_step / 1e9, 4),
         "step_gbs": round(algo_step / t_step / 1e9, 1),
         "step_frac_of_hbm": round(algo_step / t_step / 1e9 / peak, 4),
-        "roofline": {"bound": "hbm", "kernel": "decode_partial_kernel<fused>", "achieved": round(achieved, 1),
+        "roofline": {"bound": "hbm", "kernel": "decode_mma_kernel<G, fused>", "achieved": round(achieved, 1),
                      "peak": peak, "unit": "GB/s", "frac": round(achieved / peak, 4), "peak_source": src,
                      "frac_of_nominal_8000": round(achieved / 8000.0, 4),
                      "bytes_per_launch": int(part_bytes), "avg_launch_us": round(t_launch * 1e6, 2),

@@ -1,7 +1,7 @@
 // Host side of the C ABI declared in include/dkv.h: argument checks, the plan
 // object, device allocations and kernel launches. No computation of the path
-// happens here; every step runs in the kernels of dkv_map.cu, dkv_compact.cu
-// and dkv_decode.cu.
+// happens here; every step runs in the kernels of dkv_map.cu, dkv_compact.cu,
+// dkv_decode_mma.cu and dkv_decode.cu.
 #include "dkv.h"
 #include "dkv_internal.cuh"
 
@@ -32,6 +32,7 @@ struct dkv_plan {
     int32_t* d_slab_count = nullptr;  // [B*H_kv][G] arrival counters of the fused combine
     dkv::DecodeConfig cfg{};
     int64_t slots = 0;
+    int use_mma = 0;  // tensor-core decode kernel (needs the cache's row count for its tensor maps)
 };
 
 namespace {
@@ -126,7 +127,8 @@ dkv_status check_shape(const dkv_shape* s, int32_t B)
 dkv_status finish_plan(dkv_plan* p)
 {
     cudaGetDevice(&p->device);
-    cudaError_t e = dkv::decode_config(p->G, p->B, &p->cfg);
+    p->use_mma = p->total_rows >= 1 && p->total_rows <= dkv::kMaxMmaRows;
+    cudaError_t e = p->use_mma ? dkv::decode_config_mma(p->G, p->B, &p->cfg) : dkv::decode_config(p->G, p->B, &p->cfg);
     if (e != cudaSuccess) return cuda_fail(e, "decode_config");
     p->slots = (int64_t)p->cfg.nctas + p->B * p->s.H_kv;
     dkv_status st = dalloc(&p->d_work, (size_t)dkv::decode_workspace_floats(p->cfg, p->G, p->B * p->s.H_kv),
@@ -457,6 +459,22 @@ dkv_status decode_args(const dkv_plan* p, int32_t layer, const void* q, const vo
     return DKV_OK;
 }
 
+// The split-K pass of one layer, with the merge fused in or not.
+dkv_status launch_split_k(const dkv_plan* p, const dkv::DecodeArgs& a, bool fused, cudaStream_t stream)
+{
+    const char* what = fused ? "decode kernel" : "decode partial kernel";
+    if (p->use_mma) {
+        dkv::CacheMaps maps;
+        const cudaError_t e = dkv::make_cache_maps(a.Kc, a.Vc, p->total_rows, &maps);
+        if (e != cudaSuccess) return cuda_fail(e, "tensor maps of the packed caches");
+        return launched(fused ? dkv::launch_decode_mma_fused(a, maps, p->cfg, stream)
+                              : dkv::launch_decode_mma_partial(a, maps, p->cfg, stream),
+                        what);
+    }
+    return launched(fused ? dkv::launch_decode_fused(a, p->cfg, stream) : dkv::launch_decode_partial(a, p->cfg, stream),
+                    what);
+}
+
 }  // namespace
 
 dkv_status dkv_decode_attn(const dkv_plan* p, int32_t layer, const void* q, const void* k_new, const void* v_new,
@@ -467,7 +485,7 @@ dkv_status dkv_decode_attn(const dkv_plan* p, int32_t layer, const void* q, cons
     dkv_status st = decode_args(p, layer, q, k_new, v_new, k_new != nullptr, n_appended, Kc, Vc, scale, out,
                                 true, true, &a);
     if (st != DKV_OK) return st;
-    st = launched(dkv::launch_decode_fused(a, p->cfg, stream), "decode kernel");
+    st = launch_split_k(p, a, true, stream);
     return st == DKV_OK ? ok() : st;
 }
 
@@ -479,7 +497,7 @@ dkv_status dkv_decode_partial(const dkv_plan* p, int32_t layer, const void* q, c
     dkv_status st = decode_args(p, layer, q, k_new, v_new, k_new != nullptr, n_appended, Kc, Vc, scale,
                                 nullptr, true, false, &a);
     if (st != DKV_OK) return st;
-    st = launched(dkv::launch_decode_partial(a, p->cfg, stream), "decode partial kernel");
+    st = launch_split_k(p, a, false, stream);
     return st == DKV_OK ? ok() : st;
 }
 

@@ -20,7 +20,7 @@
 // earlier goes to a per-warp record (first slab) or straight to the CTA's slot
 // (a slab wholly inside the warp's range). Warps do not wait for each other
 // until their ranges are done; then the CTA merges the states that share a slab.
-#include "dkv_internal.cuh"
+#include "dkv_decode_common.cuh"
 
 #include <math.h>
 
@@ -29,169 +29,9 @@
 namespace dkv {
 namespace {
 
-constexpr unsigned kFull = 0xffffffffu;
-constexpr int kMaxB = 512;
-constexpr int kWaitSpins = 1 << 22;  // bound on mbarrier polls (each poll may suspend)
-constexpr float kSlack = 8.f;        // lazy-rescale threshold of the online softmax (log2 units)
-constexpr int PRE = 1;               // tiles a warp fetches before waiting for the previous kernel
-
-// ------------------------------------------------------------ PTX helpers
-__device__ __forceinline__ uint32_t smem_u32(const void* p)
-{
-    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count)
-{
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes)
-{
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
-                 : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
-{
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-
-// Bounded wait: false when the phase did not complete within kWaitSpins polls.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity)
-{
-    for (int i = 0; i < kWaitSpins; ++i)
-        if (mbar_try_wait(bar, parity)) return true;
-    return false;
-}
-
-__device__ __forceinline__ uint64_t evict_first_policy()
-{
-    uint64_t pol;
-    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
-    return pol;
-}
-
-__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes,
-                                         uint32_t bar, uint64_t pol)
-{
-    asm volatile(
-        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-        " [%0], [%1], %2, [%3], %4;" ::"r"(dst),
-        "l"(src), "r"(bytes), "r"(bar), "l"(pol)
-        : "memory");
-}
-
-// Programmatic dependent launch: let the next kernel in the stream start its
-// prologue, and wait for the previous kernel's results before reading them.
-__device__ __forceinline__ void pdl_launch_dependents()
-{
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-}
-
-__device__ __forceinline__ void pdl_wait()
-{
-    asm volatile("griddepcontrol.wait;" ::: "memory");
-}
-
-__device__ __forceinline__ void fence_proxy_async_smem()
-{
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-
-// ------------------------------------------------------------ partition
-// Per-call sequence table in shared memory: NA[b] = rows already appended
-// (clamped to the reserve), NP[b] = exclusive prefix over b of the extra rows
-// e_b = NA[b] + (this call appends to b ? 1 : 0). Layer rows fit in int32.
-struct SeqTable {
-    int32_t* NA;  // [B]
-    int32_t* NP;  // [B+1]
-};
-
-__device__ void build_seq_table(const DecodeArgs& a, SeqTable t, bool report)
-{
-    // Called by one full warp.
-    const int lane = threadIdx.x & 31;
-    int carry = 0;
-    for (int b0 = 0; b0 < a.B; b0 += 32) {
-        const int b = b0 + lane;
-        int na = 0, e = 0;
-        if (b < a.B) {
-            const int raw = a.n_app ? a.n_app[b] : 0;
-            na = min(max(raw, 0), a.reserve);
-            const bool app = a.append && raw >= 0 && raw < a.reserve;
-            if (a.append && !app && report) atomicOr(a.status, 0x1 /* DKV_DEV_APPEND_OVERFLOW */);
-            e = na + (app ? 1 : 0);
-            t.NA[b] = na;
-        }
-        int incl = e;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int v = __shfl_up_sync(kFull, incl, o);
-            if (lane >= o) incl += v;
-        }
-        if (b < a.B) t.NP[b] = carry + incl - e;
-        carry += __shfl_sync(kFull, incl, 31);
-    }
-    if (lane == 0) t.NP[a.B] = carry;
-}
-
-// First layer row of slab h (h in [0, B*Hkv]) within this call.
-__device__ __forceinline__ int slab_start(const DecodeArgs& a, const SeqTable& t, int h)
-{
-    const int b = h / a.Hkv, g = h - b * a.Hkv;
-    int p = (int)(a.ioff[h] - a.ioff[0]) + a.Hkv * t.NP[b];
-    if (g) p += g * (t.NP[b + 1] - t.NP[b]);
-    return p;
-}
-
-__device__ __forceinline__ int part_start(int w, int R, int P)
-{
-    // floor(w R / P) without a 64-bit division: R = q P + r, so w R / P = w q + w r / P,
-    // and w r < P^2 fits 32 bits (P is a CTA count).
-    const unsigned q = (unsigned)R / (unsigned)P, r = (unsigned)R - q * (unsigned)P;
-    return (int)((unsigned)w * q + ((unsigned)w * r) / (unsigned)P);
-}
-
-// Largest part w with part_start(w) <= x, for 0 <= x < R.
-__device__ __forceinline__ int part_of(int x, int R, int P)
-{
-    int w = min(P - 1, (int)((float)x * ((float)P / (float)R)));  // estimate, then exact steps
-    while (w + 1 < P && part_start(w + 1, R, P) <= x) ++w;
-    while (w > 0 && part_start(w, R, P) > x) --w;
-    return w;
-}
-
-// Last slab h in [0, NHl) with slab_start(h) <= x.
-__device__ int slab_containing(const DecodeArgs& a, const SeqTable& t, int NHl, int x)
-{
-    int lo = 0, hi = NHl - 1;
-    while (lo < hi) {
-        const int mid = (lo + hi + 1) >> 1;
-        if (slab_start(a, t, mid) <= x)
-            lo = mid;
-        else
-            hi = mid - 1;
-    }
-    return lo;
-}
+// (constants, PTX helpers, partition and merge helpers: dkv_decode_common.cuh)
 
 // ------------------------------------------------------------ partial kernel
-__device__ __forceinline__ float ex2(float x)
-{
-    float y;
-    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-    return y;
-}
-
 // Packed pair of fp32 values (one 64-bit register pair) for fma.rn.f32x2.
 __device__ __forceinline__ uint64_t pk(float lo, float hi)
 {
@@ -274,48 +114,6 @@ struct PK {
     static_assert(TR % RPS == 0 && 32 % TR == 0, "tile geometry");
     static_assert(kStateFloats * 4 <= NS * kStageBytes, "a warp's final state fits in its ring");
 };
-
-// Tile cursor of one warp over its row range, with the current slab's constants.
-struct Cursor {
-    int h;         // slab; == hend when exhausted
-    int s0, s1;    // the warp's rows of this slab, [s0, s1) (layer rows)
-    int p0;        // slab_start(h)
-    int x;         // first row of the current tile
-    int n_h;       // rows of the slab in this call
-    int app;       // this call appends the slab's last row from k_new/v_new
-    int64_t base;  // off[h]: cache row of the slab's first row
-};
-
-__device__ __forceinline__ void cursor_seek(Cursor& cu, const DecodeArgs& a, const SeqTable& t, int hend, int wA,
-                                            int wB)
-{
-    while (cu.h < hend) {
-        cu.p0 = slab_start(a, t, cu.h);
-        const int p1 = slab_start(a, t, cu.h + 1);
-        cu.s0 = max(wA, cu.p0);
-        cu.s1 = min(wB, p1);
-        if (cu.s0 < cu.s1) {
-            const int b = cu.h / a.Hkv;
-            const int e = t.NP[b + 1] - t.NP[b];
-            cu.n_h = a.len[cu.h] + e;
-            cu.app = (a.append && e > t.NA[b]) ? 1 : 0;
-            cu.base = a.off[cu.h];
-            cu.x = cu.s0;
-            return;
-        }
-        ++cu.h;
-    }
-}
-
-template <int TR>
-__device__ __forceinline__ void cursor_next(Cursor& cu, const DecodeArgs& a, const SeqTable& t, int hend, int wA,
-                                            int wB)
-{
-    cu.x += TR;
-    if (cu.x < cu.s1) return;
-    ++cu.h;
-    cursor_seek(cu, a, t, hend, wA, wB);
-}
 
 // Per-warp running state of one slab segment.
 template <class C>
@@ -441,81 +239,6 @@ __device__ __forceinline__ void tile_compute(State<C>& S, const uint64_t (&q2)[C
 #pragma unroll
             for (int i = 0; i < DPL / 2; ++i) S.o2[j][i] = fma2(pp[j], v2[i], S.o2[j][i]);
     }
-}
-
-// Number of CTAs whose row range overlaps [p0, p1) (p0 < p1), and the first and
-// last of them.
-__device__ __forceinline__ int ctas_of_slab(int p0, int p1, int R, int P, int* c0_out, int* c1_out)
-{
-    const int c0 = part_of(p0, R, P), c1 = part_of(p1 - 1, R, P);
-    int n = c1 - c0 + 1;
-    if (R < P) {  // some CTAs have no rows (never when every CTA gets at least one)
-        n = 0;
-        for (int cc = c0; cc <= c1; ++cc) n += part_start(cc, R, P) < part_start(cc + 1, R, P) ? 1 : 0;
-    }
-    *c0_out = c0;
-    *c1_out = c1;
-    return n;
-}
-
-// out[b][g*G + j] = O / L for the group's heads; O, L per head j for the lane's 4 dims.
-template <int G>
-__device__ __forceinline__ void write_out(const DecodeArgs& a, int b, int g, int j, float4 O, float L, int lane)
-{
-    const float inv = L > 0.f ? 1.f / L : 0.f;
-    float4* dst = reinterpret_cast<float4*>(a.out + ((int64_t)b * a.H + g * G + j) * kHeadDim);
-    dst[lane] = make_float4(O.x * inv, O.y * inv, O.z * inv, O.w * inv);
-}
-
-// Fused combine of head j of slab h by one warp of the last CTA to finish the
-// slab: the CTA partials in slots c + h, c in [c0, c1]. Lanes read the (m, l) of
-// 32 partials at a time in parallel; the weighted sum of o then loads four
-// partials at a time, all four loads in flight before any is used. Partials come
-// from other SMs: L2 loads.
-template <int G>
-__device__ void merge_slab_head(const DecodeArgs& a, int h, int j, int c0, int c1, int R, int lane)
-{
-    // Every lane loads the (m, l) and its 4 dims of o of KB partials at once (one
-    // L2 round per batch), then merges them in registers; batches chain online.
-    constexpr int KB = 16;
-    const int b = h / a.Hkv, g = h - b * a.Hkv;
-    const int P = a.nctas;
-    const bool all_live = R >= P;  // every CTA has rows
-    float M = -INFINITY, L = 0.f;
-    float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int k0 = c0; k0 <= c1; k0 += KB) {
-        float2 ml[KB];
-        float4 v[KB];
-#pragma unroll
-        for (int u = 0; u < KB; ++u) {
-            const int cc = k0 + u;
-            const bool ok = cc <= c1 && (all_live || part_start(cc, R, P) < part_start(cc + 1, R, P));
-            const int64_t sj = ((int64_t)cc + h) * G + j;
-            ml[u] = ok ? __ldcg(reinterpret_cast<const float2*>(a.work_ml + sj * 2)) : make_float2(-INFINITY, 0.f);
-            v[u] = ok ? __ldcg(reinterpret_cast<const float4*>(a.work_o + sj * kHeadDim) + lane)
-                      : make_float4(0.f, 0.f, 0.f, 0.f);
-        }
-        float Mb = M;
-#pragma unroll
-        for (int u = 0; u < KB; ++u) Mb = fmaxf(Mb, ml[u].x);
-        const float fo = (M == -INFINITY) ? 0.f : ex2(M - Mb);
-        L *= fo;
-        O.x *= fo;
-        O.y *= fo;
-        O.z *= fo;
-        O.w *= fo;
-#pragma unroll
-        for (int u = 0; u < KB; ++u) {
-            const float f = (ml[u].x == -INFINITY) ? 0.f : ex2(ml[u].x - Mb);
-            L = fmaf(f, ml[u].y, L);
-            O.x = fmaf(f, v[u].x, O.x);
-            O.y = fmaf(f, v[u].y, O.y);
-            O.z = fmaf(f, v[u].z, O.z);
-            O.w = fmaf(f, v[u].w, O.w);
-        }
-        M = Mb;
-    }
-    write_out<G>(a, b, g, j, O, L, lane);
 }
 
 // Final answer of a slab held by one warp: out = o / l for the lane's dims
@@ -807,78 +530,7 @@ __global__ void __launch_bounds__(C::NW * 32, 1) decode_partial_kernel(const Dec
     __syncthreads();
     pdl_wait();  // the merges write the workspace and out: the previous kernel must be done with them
 
-    // Entry e (lane e) is the first (even e) or last (odd e) slab of warp e/2, -1 if
-    // none; entries list their slabs in non-decreasing order. Task t = (slab #t/G,
-    // head t%G) for the distinct slabs; warp w takes tasks w, w+NW, ...
-    static_assert(2 * NW <= 32, "one entry per lane");
-    const int h_e = (lane < 2 * NW) ? ((lane & 1) ? seg_last[lane >> 1] : seg_first[lane >> 1]) : -1;
-    int prev = -1;  // slab of the nearest valid entry before this one
-#pragma unroll
-    for (int f = 0; f < 2 * NW; ++f) {
-        const int hf = __shfl_sync(kFull, h_e, f);
-        if (f < lane && hf >= 0) prev = hf;
-    }
-    const unsigned fresh = __ballot_sync(kFull, h_e >= 0 && h_e != prev);
-    const int nslab = __popc(fresh);
-    for (int t = warp; t < nslab * G; t += NW) {
-        const int si = t / G, j = t - si * G;
-        unsigned m = fresh;
-        for (int k = 0; k < si; ++k) m &= m - 1;
-        const int h = __shfl_sync(kFull, h_e, __ffs(m) - 1);
-        const unsigned same = __ballot_sync(kFull, h_e == h);
-        int c0h = 0, c1h = 0;
-        const int nct =
-            FUSED ? ctas_of_slab(slab_start(a, tab, h), slab_start(a, tab, h + 1), R, a.nctas, &c0h, &c1h) : 0;
-        float M = -INFINITY;
-#pragma unroll
-        for (int f = 0; f < 2 * NW; ++f) {
-            if (!((same >> f) & 1u)) continue;
-            const int w = f >> 1;
-            const float* ml = (f & 1) ? reinterpret_cast<const float*>(smem + w * NS * C::kStageBytes) + G * kHeadDim
-                                      : a.warp_ml + ((int64_t)c * NW + w) * G * 2;
-            M = fmaxf(M, ml[2 * j]);
-        }
-        float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
-        float L = 0.f;
-#pragma unroll
-        for (int f = 0; f < 2 * NW; ++f) {
-            if (!((same >> f) & 1u)) continue;
-            const int w = f >> 1;
-            const float* ob = (f & 1) ? reinterpret_cast<const float*>(smem + w * NS * C::kStageBytes)
-                                      : a.warp_o + ((int64_t)c * NW + w) * G * kHeadDim;
-            const float* ml = (f & 1) ? ob + G * kHeadDim : a.warp_ml + ((int64_t)c * NW + w) * G * 2;
-            const float2 mlj = *reinterpret_cast<const float2*>(ml + 2 * j);
-            const float fct = (mlj.x == -INFINITY) ? 0.f : ex2(mlj.x - M);
-            L = fmaf(mlj.y, fct, L);
-            const float4 v = reinterpret_cast<const float4*>(ob + j * kHeadDim)[lane];
-            O.x = fmaf(v.x, fct, O.x);
-            O.y = fmaf(v.y, fct, O.y);
-            O.z = fmaf(v.z, fct, O.z);
-            O.w = fmaf(v.w, fct, O.w);
-        }
-        if (FUSED && nct == 1) {
-            write_out<G>(a, h / a.Hkv, h % a.Hkv, j, O, L, lane);  // the slab lies wholly in this CTA
-            continue;
-        }
-        const int64_t slot = (int64_t)c + h;
-        reinterpret_cast<float4*>(a.work_o + (slot * G + j) * kHeadDim)[lane] = O;
-        if (lane == 0) *reinterpret_cast<float2*>(a.work_ml + (slot * G + j) * 2) = make_float2(M, L);
-        if (!FUSED) continue;
-        // Count this CTA in for (slab, head): release of the partial just written,
-        // and, for the last CTA, acquire of the others' before merging them.
-        __syncwarp();
-        int last = 0;
-        if (lane == 0) {
-            int32_t* ctr = a.slab_count + (int64_t)h * G + j;
-            int old;
-            asm volatile("atom.add.acq_rel.gpu.s32 %0, [%1], 1;" : "=r"(old) : "l"(ctr) : "memory");
-            last = (old == nct - 1) ? 1 : 0;
-            if (last) *ctr = 0;  // ready for the next call
-        }
-        last = __shfl_sync(kFull, last, 0);
-        __syncwarp();
-        if (last) merge_slab_head<G>(a, h, j, c0h, c1h, R, lane);
-    }
+    cta_tail<G, NW, FUSED>(a, tab, smem, NS * C::kStageBytes, seg_first, seg_last, c, R, warp, lane);
 }
 
 // ------------------------------------------------------------ combine kernel
@@ -983,25 +635,6 @@ __global__ void advance_kernel(int32_t* n_app, int B, int reserve, int32_t* stat
 #endif
 template <int G>
 using PKFor = typename std::conditional<(G <= 4), PK<G, DKV_CFG_SMALL_G>, PK<G, DKV_CFG_LARGE_G>>::type;
-
-// Launch with programmatic stream serialization: the kernel may start while the
-// previous kernel in the stream drains, and waits (griddepcontrol.wait) before
-// it reads that kernel's results.
-template <class K>
-cudaError_t launch_pdl(K kernel, int grid, int block, int smem, cudaStream_t st, const DecodeArgs& a)
-{
-    cudaLaunchConfig_t lc = {};
-    lc.gridDim = dim3(grid);
-    lc.blockDim = dim3(block);
-    lc.dynamicSmemBytes = smem;
-    lc.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    lc.attrs = attr;
-    lc.numAttrs = 1;
-    return cudaLaunchKernelEx(&lc, kernel, a);
-}
 
 template <int G, bool FUSED>
 cudaError_t launch_partial_g(const DecodeArgs& a, const DecodeConfig& cfg, cudaStream_t st)

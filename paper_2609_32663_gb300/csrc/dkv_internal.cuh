@@ -3,6 +3,7 @@
 #pragma once
 
 #include <cstdint>
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 namespace dkv {
@@ -92,6 +93,21 @@ cudaError_t launch_decode_partial(const DecodeArgs& a, const DecodeConfig& cfg, 
 // the slab's partials and writes out (uses a.slab_count).
 cudaError_t launch_decode_fused(const DecodeArgs& a, const DecodeConfig& cfg, cudaStream_t st);
 cudaError_t launch_decode_combine(const DecodeArgs& a, cudaStream_t st);
+
+// Tensor-core decode kernel (dkv_decode_mma.cu): the same passes with K/V tiles
+// fetched as 2-D TMA boxes through tensor maps of the packed K and V caches
+// (rows x 128 bf16, 256-byte rows). Usable while the cache has at most
+// kMaxMmaRows rows (TMA row coordinates are 32-bit).
+struct CacheMaps {
+    CUtensorMap k, v;
+};
+constexpr int64_t kMaxMmaRows = ((int64_t)1 << 31) - 16;
+cudaError_t make_cache_maps(const void* Kc, const void* Vc, int64_t rows, CacheMaps* maps);
+cudaError_t decode_config_mma(int G, int B, DecodeConfig* cfg);
+cudaError_t launch_decode_mma_partial(const DecodeArgs& a, const CacheMaps& maps, const DecodeConfig& cfg,
+                                      cudaStream_t st);
+cudaError_t launch_decode_mma_fused(const DecodeArgs& a, const CacheMaps& maps, const DecodeConfig& cfg,
+                                    cudaStream_t st);
 cudaError_t launch_advance(int32_t* n_app, int B, int reserve, int32_t* status, cudaStream_t st);
 
 }  // namespace dkv
