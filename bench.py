@@ -43,9 +43,9 @@ from paper_2609_32663_gb300 import inputs as I  # noqa: E402
 DECODE_TRAFFIC = {
     "sources": ("paper_2609_32663_gb300/csrc/dkv_decode_mma.cu", "paper_2609_32663_gb300/csrc/dkv_decode_common.cuh",
                 "paper_2609_32663_gb300/csrc/dkv_internal.cuh"),
-    "sha256": None,  # no capture of this kernel version yet
-    "dram_bytes": None,
-    "algorithmic_bytes": None,
+    "sha256": "e0fcc32eeb459b8cfebbd09ff6d198af4aaa2382d8273c96a5100378b27de44e",
+    "dram_bytes": 194_380_288 + 3_380_480,
+    "algorithmic_bytes": 376_646 * 512 + 32 * 128 * (2 + 4),
     "capture": "profiles/decode_mma_llama8b-128k-l4.md",
 }
 

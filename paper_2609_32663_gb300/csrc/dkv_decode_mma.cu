@@ -26,6 +26,7 @@
 #include <math.h>
 
 #include <mutex>
+#include <type_traits>
 
 namespace dkv {
 namespace {
@@ -48,11 +49,18 @@ struct MK {
     static_assert(G * (kHeadDim + 2) * 4 <= kWarpRing, "a warp's final state fits in its ring");
 };
 
-#ifndef DKV_MMA_CFG
-#define DKV_MMA_CFG 3, 8
+// Stages per warp, warps per CTA. The ring holds 192 KB per SM either way; more
+// warps hide more of a tile's latency chain (8 dependent score MMAs, softmax,
+// 16 output MMAs), and at the end of a pass the CTA's (slab, head) merge tasks
+// spread over more warps, which counts for G > 4 (G tasks per slab).
+#ifndef DKV_MMA_CFG_SMALL_G
+#define DKV_MMA_CFG_SMALL_G 2, 12
+#endif
+#ifndef DKV_MMA_CFG_LARGE_G
+#define DKV_MMA_CFG_LARGE_G 1, 16
 #endif
 template <int G>
-using MKFor = MK<G, DKV_MMA_CFG>;
+using MKFor = typename std::conditional<(G <= 4), MK<G, DKV_MMA_CFG_SMALL_G>, MK<G, DKV_MMA_CFG_LARGE_G>>::type;
 
 // ------------------------------------------------------------ PTX wrappers
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar,
