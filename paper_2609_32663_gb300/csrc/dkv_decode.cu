@@ -107,7 +107,7 @@ struct PK {
     static constexpr int kRingBytes = NW * NS * kStageBytes;
     static constexpr int kScratchBytes = NW * kWarpScratch;
     static constexpr int kBarBytes = NW * NS * 8;
-    static constexpr int kMetaBytes = NW * 2 * 4 + 16;  // first/last slab of each warp
+    static constexpr int kMetaBytes = NW * 6 * 4 + 16;  // first/last slab of each warp, their row bounds
     static constexpr int kFixedBytes = kRingBytes + kScratchBytes + kBarBytes + kMetaBytes;
     static constexpr int kStateFloats = G * (kHeadDim + 2);
     static int bytes(int B) { return kFixedBytes + (2 * B + 1) * 4; }
@@ -328,6 +328,8 @@ __global__ void __launch_bounds__(C::NW * 32, 1) decode_partial_kernel(const Dec
     tab.NP = tab.NA + a.B;
     int32_t* seg_first = reinterpret_cast<int32_t*>(smem + C::kRingBytes + C::kScratchBytes + C::kBarBytes);
     int32_t* seg_last = seg_first + NW;
+    int32_t* seg_p0 = seg_first + 2 * NW;  // [2 NW] layer rows [p0, p1) of entry 2 w (first) / 2 w + 1 (last)
+    int32_t* seg_p1 = seg_first + 4 * NW;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int sl = lane % LPR;
@@ -429,6 +431,7 @@ __global__ void __launch_bounds__(C::NW * 32, 1) decode_partial_kernel(const Dec
 
         while (cp.h < hend && !dead) {
             const int h = cp.h;
+            const int p0h = cp.p0, p1h = cp.p0 + cp.n_h;  // the slab's layer rows
             const int b = h / a.Hkv, g = h - b * a.Hkv;
             // q of the group, unscaled, as packed fp32 pairs of the lane's dims.
             uint64_t q2[G][DPL / 2];
@@ -496,11 +499,19 @@ __global__ void __launch_bounds__(C::NW * 32, 1) decode_partial_kernel(const Dec
             finish_state<C>(S, l_all);
             if (h == hlast) {
                 have_last = true;  // merged with the other warps at the end
-                if (lane == 0) seg_last[warp] = h;
+                if (lane == 0) {
+                    seg_last[warp] = h;
+                    seg_p0[2 * warp + 1] = p0h;
+                    seg_p1[2 * warp + 1] = p1h;
+                }
             } else if (h == hfirst) {
                 const int64_t rec = (int64_t)c * NW + warp;  // this slab continues in an earlier warp
                 store_state<C>(S, l_all, a.warp_o + rec * G * kHeadDim, a.warp_ml + rec * G * 2, lane);
-                if (lane == 0) seg_first[warp] = h;
+                if (lane == 0) {
+                    seg_first[warp] = h;
+                    seg_p0[2 * warp] = p0h;
+                    seg_p1[2 * warp] = p1h;
+                }
             } else if (FUSED) {
                 write_out_state<C>(a, S, l_all, b, g, lane);  // the whole slab lies in this warp's range
             } else {
@@ -530,7 +541,7 @@ __global__ void __launch_bounds__(C::NW * 32, 1) decode_partial_kernel(const Dec
     __syncthreads();
     pdl_wait();  // the merges write the workspace and out: the previous kernel must be done with them
 
-    cta_tail<G, NW, FUSED>(a, tab, smem, NS * C::kStageBytes, seg_first, seg_last, c, R, warp, lane);
+    cta_tail<G, NW, FUSED>(a, smem, NS * C::kStageBytes, seg_first, c, R, warp, lane);
 }
 
 // ------------------------------------------------------------ combine kernel

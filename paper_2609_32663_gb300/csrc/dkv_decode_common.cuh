@@ -145,13 +145,17 @@ __device__ __forceinline__ int part_start(int w, int R, int P)
     return (int)((unsigned)w * q + ((unsigned)w * r) / (unsigned)P);
 }
 
-// Largest part w with part_start(w) <= x, for 0 <= x < R.
+// Largest part w with part_start(w) <= x, for 0 <= x < R. part_start(w) <= x
+// exactly when w R < (x + 1) P, so w = floor(((x + 1) P - 1) / R): a float
+// estimate of that quotient, then exact integer steps (a chain of integer
+// divisions here would put ~0.5 us on the end of every launch).
 __device__ __forceinline__ int part_of(int x, int R, int P)
 {
-    int w = min(P - 1, (int)((float)x * ((float)P / (float)R)));  // estimate, then exact steps
-    while (w + 1 < P && part_start(w + 1, R, P) <= x) ++w;
-    while (w > 0 && part_start(w, R, P) > x) --w;
-    return w;
+    const int64_t num = (int64_t)(x + 1) * P - 1;
+    int w = (int)((float)num * __fdividef(1.f, (float)R));
+    while ((int64_t)(w + 1) * R <= num) ++w;
+    while (w > 0 && (int64_t)w * R > num) --w;
+    return min(w, P - 1);
 }
 
 // Last slab h in [0, NHl) with slab_start(h) <= x.
@@ -243,19 +247,18 @@ __device__ __forceinline__ void write_out(const DecodeArgs& a, int b, int g, int
 }
 
 // Fused combine of head j of slab h by one warp of the last CTA to finish the
-// slab: the CTA partials in slots c + h, c in [c0, c1]. Lanes read the (m, l) of
-// 32 partials at a time in parallel; the weighted sum of o then loads four
-// partials at a time, all four loads in flight before any is used. Partials come
-// from other SMs: L2 loads.
-template <int G>
+// slab: the CTA partials in slots c + h, c in [c0, c1], which come from other
+// SMs (L2 loads). Every lane loads the (m, l) and its 4 dims of o of KB partials
+// at once, then merges them in registers; batches chain online. Measured: a
+// load round at the end of a launch takes ~1.5 us and grows with the bytes in
+// flight, so one round of 20-24 partials costs more than two smaller ones; of
+// 8, 10, 12, 16, 20 and 24, KB = 12 was fastest.
+template <int G, int KB>
 __device__ void merge_slab_head(const DecodeArgs& a, int h, int j, int c0, int c1, int R, int lane)
 {
-    // Every lane loads the (m, l) and its 4 dims of o of KB partials at once (one
-    // L2 round per batch), then merges them in registers; batches chain online.
-    constexpr int KB = 16;
     const int b = h / a.Hkv, g = h - b * a.Hkv;
     const int P = a.nctas;
-    const bool all_live = R >= P;  // every CTA has rows
+    const bool all_live = R >= P;
     float M = -INFINITY, L = 0.f;
     float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int k0 = c0; k0 <= c1; k0 += KB) {
@@ -294,7 +297,10 @@ __device__ void merge_slab_head(const DecodeArgs& a, int h, int j, int c0, int c
 }
 
 // End of one CTA's split-K pass, after its warps' ranges are done and a CTA
-// barrier. seg_first[w] / seg_last[w]: first / last slab of warp w (-1 if none);
+// barrier. meta: seg_first[NW], seg_last[NW] (first / last slab of warp w, -1 if
+// none), then the layer rows [p0, p1) of each entry (2 w: first, 2 w + 1: last)
+// as p0[2 NW], p1[2 NW], recorded while streaming so the end of the pass reads
+// no plan metadata from global memory;
 // the first slab's state is in the warp record (c, w) of warp_o / warp_ml, the
 // last slab's in warp w's own ring at ring + w * warp_ring_bytes (o[G][128] then
 // (m, l)[G]). The states of each slab are merged; a slab wholly inside this CTA
@@ -302,14 +308,19 @@ __device__ void merge_slab_head(const DecodeArgs& a, int h, int j, int c0, int c
 // and, fused, counts itself in for each (slab, head): the last CTA to arrive
 // merges all CTA partials of that (slab, head).
 template <int G, int NW, bool FUSED>
-__device__ void cta_tail(const DecodeArgs& a, const SeqTable& tab, const unsigned char* ring, int warp_ring_bytes,
-                         const int32_t* seg_first, const int32_t* seg_last, int c, int R, int warp, int lane)
+__device__ void cta_tail(const DecodeArgs& a, const unsigned char* ring, int warp_ring_bytes,
+                         const int32_t* meta, int c, int R, int warp, int lane)
 {
+    const int32_t* seg_first = meta;
+    const int32_t* seg_last = meta + NW;
+    const int32_t* seg_p0 = meta + 2 * NW;
+    const int32_t* seg_p1 = meta + 4 * NW;
     // Entry e (lane e) is the first (even e) or last (odd e) slab of warp e/2, -1 if
     // none; entries list their slabs in non-decreasing order. Task t = (slab #t/G,
     // head t%G) for the distinct slabs; warp w takes tasks w, w+NW, ...
     static_assert(2 * NW <= 32, "one entry per lane");
     const int h_e = (lane < 2 * NW) ? ((lane & 1) ? seg_last[lane >> 1] : seg_first[lane >> 1]) : -1;
+    const int p0_e = h_e >= 0 ? seg_p0[lane] : 0, p1_e = h_e >= 0 ? seg_p1[lane] : 0;
     int prev = -1;  // slab of the nearest valid entry before this one
 #pragma unroll
     for (int f = 0; f < 2 * NW; ++f) {
@@ -322,11 +333,12 @@ __device__ void cta_tail(const DecodeArgs& a, const SeqTable& tab, const unsigne
         const int si = t / G, j = t - si * G;
         unsigned m = fresh;
         for (int k = 0; k < si; ++k) m &= m - 1;
-        const int h = __shfl_sync(kFull, h_e, __ffs(m) - 1);
+        const int e0 = __ffs(m) - 1;
+        const int h = __shfl_sync(kFull, h_e, e0);
+        const int hp0 = __shfl_sync(kFull, p0_e, e0), hp1 = __shfl_sync(kFull, p1_e, e0);
         const unsigned same = __ballot_sync(kFull, h_e == h);
         int c0h = 0, c1h = 0;
-        const int nct =
-            FUSED ? ctas_of_slab(slab_start(a, tab, h), slab_start(a, tab, h + 1), R, a.nctas, &c0h, &c1h) : 0;
+        const int nct = FUSED ? ctas_of_slab(hp0, hp1, R, a.nctas, &c0h, &c1h) : 0;
         float M = -INFINITY;
 #pragma unroll
         for (int f = 0; f < 2 * NW; ++f) {
@@ -375,7 +387,7 @@ __device__ void cta_tail(const DecodeArgs& a, const SeqTable& tab, const unsigne
         }
         last = __shfl_sync(kFull, last, 0);
         __syncwarp();
-        if (last) merge_slab_head<G>(a, h, j, c0h, c1h, R, lane);
+        if (last) merge_slab_head<G, 12>(a, h, j, c0h, c1h, R, lane);
     }
 }
 

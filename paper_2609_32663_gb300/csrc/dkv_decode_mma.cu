@@ -42,7 +42,7 @@ struct MK {
     static constexpr int kWarpRing = NS * kStageBytes;
     static constexpr int kRingBytes = NW * kWarpRing;
     static constexpr int kBarBytes = NW * NS * 8;
-    static constexpr int kMetaBytes = NW * 2 * 4 + 16;  // first/last slab of each warp
+    static constexpr int kMetaBytes = NW * 6 * 4 + 16;  // first/last slab of each warp, their row bounds
     static constexpr int kAlign = 1024;                  // swizzle atoms are 1024-byte aligned
     static constexpr int kFixedBytes = kRingBytes + kBarBytes + kMetaBytes;
     static int bytes(int B) { return kAlign + kFixedBytes + (2 * B + 1) * 4; }
@@ -286,6 +286,8 @@ __global__ void __launch_bounds__(MKFor<G>::NW * 32, 1)
     tab.NP = tab.NA + a.B;
     int32_t* seg_first = reinterpret_cast<int32_t*>(smem + C::kRingBytes + C::kBarBytes);
     int32_t* seg_last = seg_first + NW;
+    int32_t* seg_p0 = seg_first + 2 * NW;  // [2 NW] layer rows [p0, p1) of entry 2 w (first) / 2 w + 1 (last)
+    int32_t* seg_p1 = seg_first + 4 * NW;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int NHl = a.B * a.Hkv;
@@ -383,6 +385,7 @@ __global__ void __launch_bounds__(MKFor<G>::NW * 32, 1)
 
         while (cp.h < hend && !dead) {
             const int h = cp.h;
+            const int p0h = cp.p0, p1h = cp.p0 + cp.n_h;  // the slab's layer rows
             const int b = h / a.Hkv, g = h - b * a.Hkv;
             uint32_t qb[8][2];
             load_q<G>(a, b, g, lane, qb);
@@ -446,11 +449,19 @@ __global__ void __launch_bounds__(MKFor<G>::NW * 32, 1)
             finish_l(S, l2);
             if (h == hlast) {
                 have_last = true;  // merged with the other warps at the end
-                if (lane == 0) seg_last[warp] = h;
+                if (lane == 0) {
+                    seg_last[warp] = h;
+                    seg_p0[2 * warp + 1] = p0h;
+                    seg_p1[2 * warp + 1] = p1h;
+                }
             } else if (h == hfirst) {
                 const int64_t rec = (int64_t)c * NW + warp;  // this slab continues in an earlier warp
                 store_mma_state<G>(S, l2, a.warp_o + rec * G * kHeadDim, a.warp_ml + rec * G * 2, lane);
-                if (lane == 0) seg_first[warp] = h;
+                if (lane == 0) {
+                    seg_first[warp] = h;
+                    seg_p0[2 * warp] = p0h;
+                    seg_p1[2 * warp] = p1h;
+                }
             } else if (FUSED) {
                 write_mma_out<G>(a, S, l2, b, g, lane);  // the whole slab lies in this warp's range
             } else {
@@ -479,7 +490,7 @@ __global__ void __launch_bounds__(MKFor<G>::NW * 32, 1)
                            lane);
     __syncthreads();
     pdl_wait();  // the merges write the workspace and out: the previous kernel must be done with them
-    cta_tail<G, NW, FUSED>(a, tab, smem, C::kWarpRing, seg_first, seg_last, c, R, warp, lane);
+    cta_tail<G, NW, FUSED>(a, smem, C::kWarpRing, seg_first, c, R, warp, lane);
 }
 
 template <int G, bool FUSED>
