@@ -43,8 +43,8 @@ from paper_2609_32663_gb300 import inputs as I  # noqa: E402
 DECODE_TRAFFIC = {
     "sources": ("paper_2609_32663_gb300/csrc/dkv_decode_mma.cu", "paper_2609_32663_gb300/csrc/dkv_decode_common.cuh",
                 "paper_2609_32663_gb300/csrc/dkv_internal.cuh"),
-    "sha256": "e0fcc32eeb459b8cfebbd09ff6d198af4aaa2382d8273c96a5100378b27de44e",
-    "dram_bytes": 194_380_288 + 3_380_480,
+    "sha256": "f521f849ee27efecf3ee2e21335368568182c01b63da24a86f4fcc3537f35496",
+    "dram_bytes": 194_368_256 + 3_062_272,
     "algorithmic_bytes": 376_646 * 512 + 32 * 128 * (2 + 4),
     "capture": "profiles/decode_mma_llama8b-128k-l4.md",
 }
