@@ -61,6 +61,9 @@ def configure(L):
                                 ctypes.c_double, P, P]
     L.oracle_append.argtypes = [P, P, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                 ctypes.c_int, P, P, P, P, P]
+    L.oracle_budget.restype = ctypes.c_long
+    L.oracle_budget.argtypes = [ctypes.c_double, ctypes.c_long, ctypes.c_long, ctypes.c_long]
+    L.oracle_topk_mask.argtypes = [P, ctypes.c_long, ctypes.c_long, P]
     L.oracle_decode.restype = None
     L.oracle_decode.argtypes = [P, P, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                 ctypes.c_int, P, P, P, P, ctypes.c_double, P]
@@ -212,6 +215,23 @@ def decode(m: Mapping, layer, B, H, Hkv, q, Kc, Vc, n_rows_app=None, scale=None,
     return out
 
 
+def budget(rho, L, H, D):
+    """K_rho = round(rho L H D) of App. A.3 (round = floor(x + 1/2)); -1 for bad arguments."""
+    return lib().oracle_budget(float(rho), int(L), int(H), int(D))
+
+
+def topk_mask(P, K):
+    """Global Top-K mask of Eq. 3: uint8 array shaped like P with the K first entries
+    (larger value first, ties to the lower flat index, NaN last) set to 1."""
+    P = _c(P, np.float32)
+    flat = P.reshape(-1)
+    M = np.zeros(max(flat.size, 1), np.uint8)
+    rc = lib().oracle_topk_mask(_p(flat), flat.size, int(K), _p(M))
+    if rc != OK:
+        raise OracleError(rc, "oracle_topk_mask")
+    return M[: flat.size].reshape(P.shape)
+
+
 __all__ = ["Geometry", "Mapping", "OracleError", "distance_bin", "keep_logical",
            "keep_physical", "validate", "map_pattern", "compact", "attend", "append", "decode",
-           "OK", "ERR_INVALID_ARG", "ERR_RANGE"]
+           "budget", "topk_mask", "OK", "ERR_INVALID_ARG", "ERR_RANGE"]

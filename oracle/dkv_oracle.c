@@ -246,3 +246,52 @@ void oracle_decode(const int32_t *len, const int64_t *off, int layer, int B, int
                           out + ((size_t)b * H + (size_t)g * G) * hd, NULL);
         }
 }
+
+/*
+ * Exact retention budget (App. A.3): K_rho = round(rho * L * H * D), with round
+ * read as floor(x + 1/2). Returns -1 for rho outside [0, 1] or a negative size.
+ */
+long oracle_budget(double rho, long L, long H, long D)
+{
+    if (!(rho >= 0.0 && rho <= 1.0) || L < 0 || H < 0 || D < 0) return -1;
+    return (long)floor(rho * (double)L * (double)H * (double)D + 0.5);
+}
+
+/* The total order of the global Top-K: larger value first; equal values (and
+ * +0 / -0) by lower flat index; NaN after every number, NaNs by index. */
+static const float *g_topk_values;
+
+static int topk_before(long i, long j)
+{
+    const float a = g_topk_values[i], b = g_topk_values[j];
+    const int na = isnan(a), nb = isnan(b);
+    if (na != nb) return nb; /* the number comes first */
+    if (!na && a != b) return a > b;
+    return i < j;
+}
+
+static int topk_cmp(const void *x, const void *y)
+{
+    const long i = *(const long *)x, j = *(const long *)y;
+    if (i == j) return 0;
+    return topk_before(i, j) ? -1 : 1;
+}
+
+/*
+ * Global Top-K selection (Eq. 3, App. A.3): M[i] = 1 for the K first entries of
+ * P (n entries, flat order) in the order above, 0 for the rest. Sorts the index
+ * list with that order and marks its first K. K must lie in [0, n].
+ */
+int oracle_topk_mask(const float *P, long n, long K, uint8_t *M)
+{
+    if (n < 0 || K < 0 || K > n || (n > 0 && (!P || !M))) return ORACLE_ERR_INVALID_ARG;
+    long *order = (long *)malloc((size_t)(n > 0 ? n : 1) * sizeof(long));
+    if (!order) return ORACLE_ERR_INVALID_ARG;
+    for (long i = 0; i < n; ++i) order[i] = i;
+    g_topk_values = P;
+    qsort(order, (size_t)n, sizeof(long), topk_cmp);
+    memset(M, 0, (size_t)n);
+    for (long r = 0; r < K; ++r) M[order[r]] = 1;
+    free(order);
+    return ORACLE_OK;
+}

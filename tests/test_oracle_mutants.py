@@ -3,7 +3,8 @@
 Each case plants one mistake in a temporary copy of oracle/dkv_oracle.c (an
 off-by-one bin, a reversed distance, a wrong window edge, intersection instead of
 union, strided GQA grouping, a dropped scale, swapped operands, offsets without
-the reserve, appending at the wrong slot), builds it with the host C compiler,
+the reserve, appending at the wrong slot, Top-K ties or order reversed, a
+truncating budget), builds it with the host C compiler,
 and runs the pin suite against it: at least one pin has to fail. The real oracle
 is restored afterwards. CPU only.
 """
@@ -41,6 +42,11 @@ MUTANTS = {
                                "size_t dst = (size_t)(off[h] + len[h] + na - 1) * hd;"),
     "descending_pack": ("for (long p = 0; p < Tc[b]; ++p)",
                         "for (long p = Tc[b] - 1; p >= 0; --p)"),
+    "topk_ties_to_higher_index": ("    return i < j;\n}", "    return i > j;\n}"),
+    "topk_nan_first": ("if (na != nb) return nb; /* the number comes first */",
+                       "if (na != nb) return na;"),
+    "topk_smallest": ("if (!na && a != b) return a > b;", "if (!na && a != b) return a < b;"),
+    "budget_truncates": ("(double)D + 0.5);", "(double)D);"),
 }
 
 
@@ -52,6 +58,8 @@ def _pin_calls():
         calls.append(lambda case=case: pins.test_map_hand_worked_cases(case))
     for seed in range(6):
         calls.append(lambda seed=seed: pins.test_length_closed_form(seed))
+    for seed in range(4):
+        calls.append(lambda seed=seed: pins.test_topk_matches_pairwise_rank_definition(seed))
     for G, hd in [(1, 4), (2, 8), (4, 128), (7, 128)]:
         calls.append(lambda G=G, hd=hd: pins.test_compacted_attention_equals_masked_dense(G, hd))
     for name in ("test_memory_arithmetic_sec43_and_app_c", "test_streaming_llm_special_case",
@@ -61,7 +69,8 @@ def _pin_calls():
                  "test_single_row_returns_that_value_row", "test_identical_keys_give_mean_of_values",
                  "test_softmax_weights_sum_to_one_and_two_row_closed_form",
                  "test_default_scale_is_inverse_sqrt_head_dim",
-                 "test_append_then_decode_equals_attention_with_new_token"):
+                 "test_append_then_decode_equals_attention_with_new_token", "test_budget_rounding_app_a3",
+                 "test_topk_equals_stable_library_sort"):
         calls.append(getattr(pins, name))
     return calls
 

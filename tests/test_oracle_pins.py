@@ -345,3 +345,69 @@ def test_append_then_decode_equals_attention_with_new_token():
             np.testing.assert_allclose(got[b, g * G:(g + 1) * G], want, rtol=1e-12, atol=1e-12)
     with pytest.raises(O.OracleError):
         O.append(m, layer, B, Hkv, 3, [3] * B, new_k[0], new_v[0], Kc, Vc)
+
+
+# ---------------------------------------------------------------- exact-budget Top-K (Eq. 3, App. A.3)
+
+def test_budget_rounding_app_a3():
+    # K_rho = round(rho L H D), round read as floor(x + 1/2).
+    assert O.budget(0.35, 32, 32, 1013) == 363059  # 363059.2
+    assert O.budget(0.5, 1, 1, 5) == 3             # 2.5 rounds up
+    assert O.budget(0.5, 1, 1, 3) == 2             # 1.5 rounds up
+    assert O.budget(0.25, 28, 28, 64) == 12544     # exact
+    assert O.budget(0.0, 32, 32, 128) == 0
+    assert O.budget(1.0, 32, 32, 128) == 32 * 32 * 128
+    assert O.budget(-0.1, 1, 1, 1) == -1 and O.budget(1.1, 1, 1, 1) == -1 and O.budget(float("nan"), 1, 1, 1) == -1
+
+
+def _rank_by_definition(P):
+    """Rank of every entry under the selection order, counted pairwise: larger
+    value first, equal values (+0 == -0) by lower index, NaN after all numbers."""
+    n = len(P)
+    rank = np.zeros(n, np.int64)
+    for i in range(n):
+        for j in range(n):
+            if i == j:
+                continue
+            a, b = P[j], P[i]  # does j come before i?
+            if np.isnan(a) != np.isnan(b):
+                before = np.isnan(b)
+            elif not np.isnan(a) and a != b:
+                before = a > b
+            else:
+                before = j < i
+            rank[i] += int(before)
+    return rank
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_topk_matches_pairwise_rank_definition(seed):
+    rng = np.random.default_rng(seed)
+    n = 23
+    P = rng.choice(np.array([0.0, -0.0, 0.25, 0.5, 0.5, 0.75, 1.0, np.nan, -np.inf, np.inf], np.float32), n)
+    P[:5] = rng.random(5).astype(np.float32)
+    rank = _rank_by_definition(P)
+    assert sorted(rank.tolist()) == list(range(n))  # a total order
+    for K in range(n + 1):
+        M = O.topk_mask(P, K)
+        assert np.array_equal(M, (rank < K).astype(np.uint8)), f"K={K}"
+        assert int(M.sum()) == K
+
+
+def test_topk_equals_stable_library_sort():
+    rng = np.random.default_rng(7)
+    P = rng.random((6, 8, 37)).astype(np.float32)
+    P[1, 2, :10] = 0.5  # ties
+    flat = P.reshape(-1)
+    order = np.lexsort((np.arange(flat.size), -flat.astype(np.float64)))
+    for K in (0, 1, 100, 1776 // 2, flat.size - 1, flat.size):
+        want = np.zeros(flat.size, np.uint8)
+        want[order[:K]] = 1
+        assert np.array_equal(O.topk_mask(P, K).reshape(-1), want)
+
+
+def test_topk_bad_arguments():
+    P = np.zeros(5, np.float32)
+    for K in (-1, 6):
+        with pytest.raises(O.OracleError):
+            O.topk_mask(P, K)
