@@ -239,6 +239,38 @@ def time_compaction(env, reps=10):
     return {"gbs": algo / t / 1e9, "ms": t * 1e3, "algorithmic_bytes": algo, "reps": reps}
 
 
+def time_topk(wl, dev, reps=10):
+    """The exact-budget pattern export (dkv_topk_mask) on the workload's
+    L x H x D probabilities and on a large synthetic one, CUDA events around each
+    call (median). Algorithmic bytes: P read once + M written (5 bytes an entry);
+    the radix select streams P six times."""
+    import torch
+
+    import paper_2609_32663_gb300.dkv as dkv
+    ws = torch.empty(dkv.dkv_topk_workspace_bytes() // 4 + 1, dtype=torch.int32, device=dev)
+    out = {}
+    big = wl.with_(L=80, H=64, D=2048)
+    for tag, w in (("pattern", wl), ("large", big)):
+        P = torch.from_numpy(I.retention_probs(w)).to(dev)
+        M = torch.empty(P.shape, dtype=torch.uint8, device=dev)
+        K = dkv.dkv_budget(0.35, w.L, w.H, w.D)
+        times = []
+        for i in range(reps + 2):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            dkv.dkv_topk_mask(P, K, M, ws)
+            e1.record()
+            e1.synchronize()
+            if i >= 2:
+                times.append(e0.elapsed_time(e1) * 1e-3)
+        t = statistics.median(times)
+        n = P.numel()
+        out[tag] = {"shape": [w.L, w.H, w.D], "n": n, "K": K, "us": round(t * 1e6, 2),
+                    "algorithmic_gbs": round(5 * n / t / 1e9, 1), "streamed_gbs": round(25 * n / t / 1e9, 1),
+                    "launches": 7}
+    return out
+
+
 def step_bytes(wl, Tc_rows_per_layer, with_new=True):
     """Algorithmic bytes of one decode step: retained K/V rows (with appended
     tokens) + q read + o written + the new K/V row written."""
@@ -528,6 +560,8 @@ def run_dkv(args, dist):
                                "sample": f"fp64 scalar oracle, {layers} of {wl.L} layers of one decode step "
                                          f"({rows} rows x G={wl.G} heads), scaled x{wl.L / layers:g} to a step",
                                "cpu": cpu_model(), "nproc": os.cpu_count()}
+    if not args.profile:
+        res["pattern_export"] = time_topk(wl, dev)
     st = dkv.dkv_plan_status(env["plan"])
     res["device_status_word"] = st
     env["plan"].close()

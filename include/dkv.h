@@ -13,6 +13,9 @@
  *   dkv_decode_attn   split-K decode attention over the packed cache
  *   dkv_free          release a plan
  *
+ * and the step before them, the export of the pattern from learned retention
+ * probabilities with an exact budget (dkv_budget, dkv_topk_mask; Eq. 3).
+ *
  * Conventions used by every entry point
  *  - A "slab" is one (layer l, sequence b, KV head g); slabs are flattened as
  *    h = (l*B + b)*H_kv + g. A "row" is one token's key (or value) vector for
@@ -244,6 +247,32 @@ dkv_status dkv_decode_attn_noalloc(const dkv_shape* s, int32_t B, int32_t layer,
 
 /* Release a plan (NULL-safe). Synchronises the device before freeing. */
 void dkv_free(dkv_plan* plan);
+
+/*
+ * Exact-budget pattern export (Sec. 3.3, Eq. 3; App. A.3): learned retention
+ * probabilities P in [0,1]^{L x H x D} become the binary pattern
+ * M = TopKMask(P, K_rho) that dkv_map_pattern takes.
+ *
+ * dkv_budget     K_rho = round(rho * L * H * D) with round(x) = floor(x + 1/2)
+ *                (host only). Returns -1 when rho is outside [0, 1] or a size is
+ *                negative.
+ * dkv_topk_workspace_bytes
+ *                device workspace bytes dkv_topk_mask needs (a few KB, the same
+ *                for every n).
+ * dkv_topk_mask  P: device float [n], any layout, read in flat order.
+ *                M: device uint8 [n], written in full. M[i] = 1 for the K first
+ *                entries in this order: larger value first; equal values (+0
+ *                and -0 are equal) by lower flat index; NaN after every number.
+ *                workspace: device scratch of at least dkv_topk_workspace_bytes()
+ *                bytes, 4-byte aligned; calls that share it must be ordered.
+ *                Asynchronous on stream; allocates nothing.
+ * Errors: DKV_ERR_INVALID_ARG (n < 0 or n >= 2^31, K outside [0, n], a NULL
+ * pointer with n > 0, a small or unaligned workspace), DKV_ERR_CUDA.
+ */
+int64_t dkv_budget(double rho, int32_t L, int32_t H, int32_t D);
+int64_t dkv_topk_workspace_bytes(void);
+dkv_status dkv_topk_mask(const float* P, int64_t n, int64_t K, uint8_t* M, void* workspace,
+                         int64_t workspace_bytes, cudaStream_t stream);
 
 #ifdef __cplusplus
 }

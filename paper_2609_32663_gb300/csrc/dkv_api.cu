@@ -1,7 +1,7 @@
 // Host side of the C ABI declared in include/dkv.h: argument checks, the plan
 // object, device allocations and kernel launches. No computation of the path
 // happens here; every step runs in the kernels of dkv_map.cu, dkv_compact.cu,
-// dkv_decode_mma.cu and dkv_decode.cu.
+// dkv_decode_mma.cu, dkv_decode.cu and dkv_topk.cu.
 #include "dkv.h"
 #include "dkv_internal.cuh"
 
@@ -509,6 +509,30 @@ dkv_status dkv_decode_combine(const dkv_plan* p, int32_t layer, const int32_t* n
                                 nullptr, 1.f, out, false, true, &a);
     if (st != DKV_OK) return st;
     st = launched(dkv::launch_decode_combine(a, stream), "decode combine kernel");
+    return st == DKV_OK ? ok() : st;
+}
+
+int64_t dkv_budget(double rho, int32_t L, int32_t H, int32_t D)
+{
+    if (!(rho >= 0.0 && rho <= 1.0) || L < 0 || H < 0 || D < 0) return -1;
+    return (int64_t)std::floor(rho * (double)L * (double)H * (double)D + 0.5);
+}
+
+int64_t dkv_topk_workspace_bytes(void) { return dkv::topk_workspace_bytes(); }
+
+dkv_status dkv_topk_mask(const float* P, int64_t n, int64_t K, uint8_t* M, void* workspace,
+                         int64_t workspace_bytes, cudaStream_t stream)
+{
+    if (n < 0 || n >= ((int64_t)1 << 31)) return fail(DKV_ERR_INVALID_ARG, "n=%lld out of [0, 2^31)", (long long)n);
+    if (K < 0 || K > n) return fail(DKV_ERR_INVALID_ARG, "K=%lld out of [0, n=%lld]", (long long)K, (long long)n);
+    if (n > 0 && (!P || !M)) return fail(DKV_ERR_INVALID_ARG, "NULL P or M");
+    if (n > 0 && K > 0 && K < n) {
+        if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 3u) != 0 ||
+            workspace_bytes < dkv::topk_workspace_bytes())
+            return fail(DKV_ERR_INVALID_ARG, "workspace: need %lld bytes, 4-byte aligned",
+                        (long long)dkv::topk_workspace_bytes());
+    }
+    const dkv_status st = launched(dkv::launch_topk(P, n, K, M, workspace, stream), "top-k kernels");
     return st == DKV_OK ? ok() : st;
 }
 

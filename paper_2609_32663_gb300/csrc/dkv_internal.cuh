@@ -110,4 +110,9 @@ cudaError_t launch_decode_mma_fused(const DecodeArgs& a, const CacheMaps& maps, 
                                     cudaStream_t st);
 cudaError_t launch_advance(int32_t* n_app, int B, int reserve, int32_t* status, cudaStream_t st);
 
+// Exact-budget Top-K pattern export (dkv_topk.cu): device workspace bytes, and
+// the launches (4 histogram passes, tie count, mark) on `st`.
+int64_t topk_workspace_bytes();
+cudaError_t launch_topk(const float* P, int64_t n, int64_t K, uint8_t* M, void* workspace, cudaStream_t st);
+
 }  // namespace dkv

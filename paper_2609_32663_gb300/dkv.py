@@ -25,7 +25,8 @@ DKV_DEV_TMA_TIMEOUT = 0x2
 # Every entry point include/dkv.h declares.
 EXPORTS = ("dkv_last_error", "dkv_map_pattern", "dkv_plan_dense", "dkv_plan_query", "dkv_plan_read",
            "dkv_compact", "dkv_decode_attn", "dkv_decode_partial", "dkv_decode_combine", "dkv_advance",
-           "dkv_plan_status", "dkv_free", "dkv_decode_attn_noalloc")
+           "dkv_plan_status", "dkv_free", "dkv_decode_attn_noalloc", "dkv_budget", "dkv_topk_workspace_bytes",
+           "dkv_topk_mask")
 
 
 class DkvError(RuntimeError):
@@ -102,6 +103,12 @@ def lib(path: str | None = None):
                                           ctypes.c_float, V, V, V]
     L.dkv_free.restype = None
     L.dkv_free.argtypes = [V]
+    L.dkv_budget.restype = I64
+    L.dkv_budget.argtypes = [ctypes.c_double, I32, I32, I32]
+    L.dkv_topk_workspace_bytes.restype = I64
+    L.dkv_topk_workspace_bytes.argtypes = []
+    L.dkv_topk_mask.restype = ctypes.c_int
+    L.dkv_topk_mask.argtypes = [V, I64, I64, V, V, I64, V]
     if path is None:
         _lib = L
     return L
@@ -232,6 +239,28 @@ def dkv_plan_status(plan: Plan, clear: bool = False, stream=None) -> int:
 
 def dkv_free(plan: Plan):
     plan.close()
+
+
+def dkv_budget(rho: float, L: int, H: int, D: int) -> int:
+    """K_rho = round(rho L H D) (App. A.3); raises on bad arguments."""
+    k = lib().dkv_budget(float(rho), int(L), int(H), int(D))
+    if k < 0:
+        raise DkvError(1, "dkv_budget", f"rho={rho} L={L} H={H} D={D}")
+    return int(k)
+
+
+def dkv_topk_workspace_bytes() -> int:
+    return int(lib().dkv_topk_workspace_bytes())
+
+
+def dkv_topk_mask(P, K: int, M, workspace, stream=None):
+    """M (device uint8, same element count as P) = TopKMask(P, K) of Eq. 3."""
+    n = P.numel()
+    if M.numel() != n:
+        raise ValueError("M must have as many elements as P")
+    nbytes = workspace.numel() * workspace.element_size()
+    _check(lib().dkv_topk_mask(_ptr(P), int(n), int(K), _ptr(M), _ptr(workspace), int(nbytes), _stream(stream)),
+           "dkv_topk_mask")
 
 
 def dkv_decode_attn_noalloc(shape: Shape, B: int, layer: int, reserve_rows: int, d_len, d_off, d_ioff, q, k_new,

@@ -152,6 +152,21 @@ def profile_pattern(wl: Workload, rng: np.random.Generator) -> np.ndarray:
     return M.reshape(L, Hkv * G, D)
 
 
+def retention_probs(wl: Workload, levels: int | None = None, seed_offset: int = 0) -> np.ndarray:
+    """Synthetic learned retention probabilities P in (0, 1)^{L x H x D} (float32),
+    the input of the exact-budget export (Eq. 3): per (layer, q-head) a Beta(2, 2)
+    near/far mix w (1 - x_d) + (1 - w) x_d plus noise, squashed by a logistic.
+    With `levels`, P is rounded to that many values, which makes many ties."""
+    rng = np.random.default_rng([wl.seed, 13, seed_offset])
+    w = rng.beta(2.0, 2.0, size=(wl.L, wl.H, 1))
+    x = (np.arange(wl.D) / max(wl.D - 1, 1))[None, None, :]
+    z = 6.0 * (w * (1.0 - x) + (1.0 - w) * x - 0.5) + rng.normal(0.0, 1.0, (wl.L, wl.H, wl.D))
+    P = 1.0 / (1.0 + np.exp(-z))
+    if levels:
+        P = np.round(P * (levels - 1)) / (levels - 1)
+    return P.astype(np.float32)
+
+
 def make_pattern(wl: Workload) -> np.ndarray:
     """The workload's retention pattern M in {0,1}^{L x H x D} (uint8)."""
     rng = np.random.default_rng([wl.seed, 7])
@@ -217,6 +232,6 @@ def bf16_bits(t) -> np.ndarray:
     return t.detach().to("cpu").contiguous().view(torch.int16).numpy().view(np.uint16)
 
 
-__all__ = ["Workload", "WORKLOADS", "SINK", "RECENT", "context_lengths", "make_pattern",
+__all__ = ["Workload", "WORKLOADS", "SINK", "RECENT", "context_lengths", "make_pattern", "retention_probs",
            "topk_mask", "round_half_up", "union_bins_target", "dense_kv", "decode_inputs",
            "bf16_bits"]

@@ -114,3 +114,32 @@ def test_binding_fails_loudly_without_library(tmp_path):
     import paper_2609_32663_gb300.dkv as dkv
     with pytest.raises(RuntimeError, match="missing"):
         dkv.lib(str(tmp_path / "libdkv.so"))
+
+
+def test_budget_matches_oracle(dkvmod):
+    """dkv_budget (host arithmetic of the library) against the oracle's budget."""
+    import oracle as O
+    rng = np.random.default_rng(3)
+    cases = [(0.35, 32, 32, 1013), (0.5, 1, 1, 5), (0.5, 1, 1, 3), (0.0, 32, 32, 128), (1.0, 28, 28, 64)]
+    cases += [(float(r), int(L), int(H), int(D)) for r, L, H, D in
+              zip(rng.random(50), rng.integers(1, 80, 50), rng.integers(1, 64, 50), rng.integers(1, 2048, 50))]
+    for rho, L, H, D in cases:
+        assert dkvmod.dkv_budget(rho, L, H, D) == O.budget(rho, L, H, D), (rho, L, H, D)
+    for bad in [(-0.01, 1, 1, 1), (1.01, 1, 1, 1), (float("nan"), 1, 1, 1), (0.5, -1, 1, 1)]:
+        with pytest.raises(dkvmod.DkvError):
+            dkvmod.dkv_budget(*bad)
+
+
+def test_topk_rejects_bad_arguments(dkvmod):
+    """Argument checks run before any launch (fake device addresses are never touched)."""
+    L = dkvmod.lib()
+    ws_need = L.dkv_topk_workspace_bytes()
+    assert 0 < ws_need <= 64 * 1024
+    fake = ctypes.c_void_p(0x1000)
+    for n, K, P, M, ws, wsb in [(-1, 0, fake, fake, fake, ws_need), (1 << 31, 1, fake, fake, fake, ws_need),
+                                (10, 11, fake, fake, fake, ws_need), (10, -1, fake, fake, fake, ws_need),
+                                (10, 3, None, fake, fake, ws_need), (10, 3, fake, None, fake, ws_need),
+                                (10, 3, fake, fake, None, ws_need), (10, 3, fake, fake, fake, ws_need - 4),
+                                (10, 3, fake, fake, ctypes.c_void_p(0x1002), ws_need)]:
+        assert L.dkv_topk_mask(P, n, K, M, ws, wsb, None) == 1, (n, K)
+        assert L.dkv_last_error()
