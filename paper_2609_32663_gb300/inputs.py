@@ -71,6 +71,14 @@ WORKLOADS = {
     "llama8b-128k-l4": Workload("llama8b-128k-l4", L=4, H=32, Hkv=8, T=131072, B=1, D=128,
                                 W=_w(131072, 128), pattern="profile", rate=0.346,
                                 physical_target=0.346, outlier_frac=0.01, seed=3),
+    # Structural ablations of llama8b-128k at matched physical retention (Sec. 4.5,
+    # App. B): the same caches, patterns with parts of the structure removed.
+    # Head-only makes the most ragged slabs (whole heads or sink + recent only).
+    **{f"llama8b-128k-{k.replace('_', '-')}": Workload(f"llama8b-128k-{k.replace('_', '-')}", L=32, H=32, Hkv=8,
+                                                       T=131072, B=1, D=128, W=_w(131072, 128),
+                                                       pattern=f"ablation:{k}", rate=0.346, physical_target=0.346,
+                                                       outlier_frac=0.01, seed=3)
+       for k in ("distance_shuffled", "fully_shuffled", "head_only", "distance_only")},
     "llama8b-b16-ragged": Workload("llama8b-b16-ragged", L=32, H=32, Hkv=8, T=65536, B=16, D=64,
                                    W=_w(65536, 64), pattern="profile", rate=0.25,
                                    ragged=(8192, 65536), seed=4),
@@ -167,9 +175,91 @@ def retention_probs(wl: Workload, levels: int | None = None, seed_offset: int = 
     return P.astype(np.float32)
 
 
+# ---------------------------------------------------------------- structural ablations
+# The paper's ablations (Sec. 4.5 ablation study, App. B) compare Distance-KV
+# with patterns of matched physical KV retention that break parts of its
+# structure. These recipes derive them from a reference pattern M. The GQA union
+# count below only sizes these inputs: it counts (layer, KV head, bin) columns
+# with any query head on, i.e. physical bins at full context coverage.
+
+def _union_count(M: np.ndarray, G: int) -> int:
+    L, H, D = M.shape
+    return int(M.reshape(L, H // G, G, D).max(axis=2).sum())
+
+
+def ablate_distance_shuffled(M: np.ndarray, G: int, rng: np.random.Generator) -> np.ndarray:
+    """Per (layer, KV head) one random permutation of the D bins, applied to all
+    of its query heads: per-head counts and each group's union count are kept,
+    the distance assignment is lost."""
+    L, H, D = M.shape
+    out = np.empty_like(M)
+    for l in range(L):
+        for g in range(H // G):
+            perm = rng.permutation(D)
+            out[l, g * G:(g + 1) * G] = M[l, g * G:(g + 1) * G][:, perm]
+    return out
+
+
+def ablate_fully_shuffled(M: np.ndarray, G: int, rng: np.random.Generator) -> np.ndarray:
+    """The G-head columns M[l, gG:(g+1)G, d] permuted over all (layer, KV head,
+    bin) positions, and the heads permuted within each column: the logical count
+    and the union (physical) count are kept, every layer / head / distance
+    correspondence is lost."""
+    L, H, D = M.shape
+    cols = M.reshape(L, H // G, G, D).transpose(0, 1, 3, 2).reshape(-1, G)  # [(l, g, d)][j]
+    cols = cols[rng.permutation(cols.shape[0])]
+    cols = np.take_along_axis(cols, np.argsort(rng.random(cols.shape), axis=1), axis=1)
+    return np.ascontiguousarray(cols.reshape(L, H // G, D, G).transpose(0, 1, 3, 2).reshape(L, H, D))
+
+
+def ablate_head_only(M: np.ndarray, G: int) -> np.ndarray:
+    """One decision per query head for all its bins. Whole KV groups are kept,
+    which is what a kept head costs physically, in descending order of the
+    group's union count in M (ties to the lower index), as many as round(U / D)
+    for the union count U of M."""
+    L, H, D = M.shape
+    score = M.reshape(L, H // G, G, D).max(axis=2).sum(axis=2).reshape(-1)  # union bins per (l, g)
+    n_groups = int(np.floor(_union_count(M, G) / D + 0.5))
+    order = np.argsort(-score, kind="stable")[:n_groups]
+    keep = np.zeros(L * (H // G), np.uint8)
+    keep[order] = 1
+    return np.ascontiguousarray(np.repeat(keep.reshape(L, H // G, 1, 1), G, axis=2)
+                                .repeat(D, axis=3).reshape(L, H, D))
+
+
+def ablate_distance_only(M: np.ndarray, G: int) -> np.ndarray:
+    """One decision per (layer, bin) shared by all query heads of the layer. A
+    kept (layer, bin) costs H/G physical bins; the round(U / (H/G)) with the most
+    query heads on in M are kept (ties to the lower index)."""
+    L, H, D = M.shape
+    Hkv = H // G
+    score = M.sum(axis=1).reshape(-1)  # query heads on per (l, d)
+    n_keep = int(np.floor(_union_count(M, G) / Hkv + 0.5))
+    order = np.argsort(-score, kind="stable")[:n_keep]
+    keep = np.zeros(L * D, np.uint8)
+    keep[order] = 1
+    return np.ascontiguousarray(np.repeat(keep.reshape(L, 1, D), H, axis=1))
+
+
+ABLATIONS = ("distance_shuffled", "fully_shuffled", "head_only", "distance_only")
+
+
 def make_pattern(wl: Workload) -> np.ndarray:
     """The workload's retention pattern M in {0,1}^{L x H x D} (uint8)."""
     rng = np.random.default_rng([wl.seed, 7])
+    if wl.pattern.startswith("ablation:"):
+        kind = wl.pattern.split(":", 1)[1]
+        base = make_pattern(wl.with_(pattern="profile"))
+        arng = np.random.default_rng([wl.seed, 23])
+        if kind == "distance_shuffled":
+            return ablate_distance_shuffled(base, wl.G, arng)
+        if kind == "fully_shuffled":
+            return ablate_fully_shuffled(base, wl.G, arng)
+        if kind == "head_only":
+            return ablate_head_only(base, wl.G)
+        if kind == "distance_only":
+            return ablate_distance_only(base, wl.G)
+        raise ValueError(f"unknown ablation {kind!r}")
     if wl.pattern == "bernoulli":
         return bernoulli_pattern(wl, rng)
     if wl.pattern == "profile":
@@ -233,5 +323,7 @@ def bf16_bits(t) -> np.ndarray:
 
 
 __all__ = ["Workload", "WORKLOADS", "SINK", "RECENT", "context_lengths", "make_pattern", "retention_probs",
+           "ABLATIONS", "ablate_distance_shuffled", "ablate_fully_shuffled", "ablate_head_only",
+           "ablate_distance_only",
            "topk_mask", "round_half_up", "union_bins_target", "dense_kv", "decode_inputs",
            "bf16_bits"]

@@ -65,7 +65,9 @@ def _dense_rows(wl, om, slabs, T_stride):
 
 
 @pytest.mark.parametrize("name", ["llama8b-1layer-4k", "llama8b-32k", "llama8b-128k", "llama8b-b16-ragged",
-                                  "qwen7b-64k-b4-r20", "qwen7b-64k-b4-r35", "qwen7b-64k-b4-r50"])
+                                  "qwen7b-64k-b4-r20", "qwen7b-64k-b4-r35", "qwen7b-64k-b4-r50",
+                                  "llama8b-128k-head-only", "llama8b-128k-distance-only",
+                                  "llama8b-128k-distance-shuffled", "llama8b-128k-fully-shuffled"])
 def test_full_size_workload(name, cuda):
     import bench
     wl = I.WORKLOADS[name]
