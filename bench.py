@@ -271,6 +271,43 @@ def time_topk(wl, dev, reps=10):
     return out
 
 
+def time_multi_query(wl, env, dev, Q, steps, warmup):
+    """Q queries per sequence over the compressed cache (dkv_decode_multi), one
+    CUDA graph of L launches per step; the K/V rows are read once for all Q."""
+    import torch
+
+    import paper_2609_32663_gb300.dkv as dkv
+    g = torch.Generator(device=dev)
+    g.manual_seed(wl.seed * 1000 + 31)
+    q = torch.randn((wl.L, wl.B, Q, wl.H, wl.head_dim), generator=g, device=dev).to(torch.bfloat16)
+    out = torch.empty((wl.L, wl.B, Q, wl.H, wl.head_dim), dtype=torch.float32, device=dev)
+    n_app = torch.zeros(wl.B, dtype=torch.int32, device=dev)
+
+    def step():
+        for layer in range(wl.L):
+            dkv.dkv_decode_multi(env["plan"], layer, q[layer], Q, n_app, env["Kc"], env["Vc"], out[layer])
+
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        step()
+    torch.cuda.current_stream().wait_stream(s)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        step()
+    for _ in range(warmup):
+        graph.replay()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(steps):
+        graph.replay()
+    e1.record()
+    e1.synchronize()
+    return e0.elapsed_time(e1) * 1e-3 / steps
+
+
 def step_bytes(wl, Tc_rows_per_layer, with_new=True):
     """Algorithmic bytes of one decode step: retained K/V rows (with appended
     tokens) + q read + o written + the new K/V row written."""
@@ -562,6 +599,13 @@ def run_dkv(args, dist):
                                "cpu": cpu_model(), "nproc": os.cpu_count()}
     if not args.profile:
         res["pattern_export"] = time_topk(wl, dev)
+        mq = {}
+        for Q in sorted({1, max(1, 8 // wl.G), max(1, 16 // wl.G)}):
+            t_q = dist.max(time_multi_query(wl, env, dev, Q, min(steps, 64), warmup))
+            rows_q = sum(rows_layer)  # no appends in these calls
+            mq[f"Q{Q}"] = {"us_per_step": round(t_q * 1e6, 2), "queries_per_s": round(wl.B * Q * dist.world / t_q, 1),
+                           "gbs": round(step_bytes(wl, rows_q, with_new=False) / t_q / 1e9, 1)}
+        res["multi_query"] = mq
     st = dkv.dkv_plan_status(env["plan"])
     res["device_status_word"] = st
     env["plan"].close()

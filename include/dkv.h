@@ -188,6 +188,26 @@ dkv_status dkv_decode_attn(const dkv_plan* plan, int32_t layer, const void* q,
                            void* Kc, void* Vc, float scale, float* out, cudaStream_t stream);
 
 /*
+ * Several queries per sequence over one compressed cache (shared-context reuse,
+ * Sec. 4.1: the compressed context cache serves the queries that follow it).
+ * Each of the num_queries queries of sequence b attends, per query head, over
+ * the same rows as dkv_decode_attn without k_new: the len[h] packed rows plus
+ * the n_appended[b] rows appended so far. Nothing is appended and the queries
+ * do not see each other.
+ *
+ * q    device bf16 [B][num_queries][H][128].
+ * out  device fp32 [B][num_queries][H][128].
+ * Needs 1 <= num_queries and num_queries * G <= 16 (G = H / H_kv), and a plan
+ * whose cache has fewer than 2^31 rows. The query x head columns of a KV head
+ * are the n side of one tensor-core product per tile of 16 rows, so the K/V
+ * rows are read once for all queries. Other arguments, ordering and errors are
+ * those of dkv_decode_attn.
+ */
+dkv_status dkv_decode_multi(const dkv_plan* plan, int32_t layer, const void* q, int32_t num_queries,
+                            const int32_t* n_appended, void* Kc, void* Vc, float scale, float* out,
+                            cudaStream_t stream);
+
+/*
  * The two halves of dkv_decode_attn, for callers that schedule them apart
  * (or time them apart). dkv_decode_partial runs the split-K pass: every CTA of
  * a persistent grid takes an equal share of the layer's rows (slabs laid end to

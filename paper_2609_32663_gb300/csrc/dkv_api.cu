@@ -5,6 +5,7 @@
 #include "dkv.h"
 #include "dkv_internal.cuh"
 
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -30,8 +31,10 @@ struct dkv_plan {
     int32_t* d_status = nullptr;
     float* d_work = nullptr;    // split-K partials
     int32_t* d_slab_count = nullptr;  // [B*H_kv][G] arrival counters of the fused combine
-    dkv::DecodeConfig cfg{};
-    int64_t slots = 0;
+    dkv::DecodeConfig cfg{};        // the decode step's kernel
+    dkv::DecodeConfig cfg_multi{};  // the multi-query kernel (tensor-core plans)
+    int64_t slots = 0;              // (CTA, slab) partial slots: CTAs + slabs of a layer
+    int nctas_cap = 0, warps_cap = 0, cols_cap = 0;  // workspace sized for these
     int use_mma = 0;  // tensor-core decode kernel (needs the cache's row count for its tensor maps)
 };
 
@@ -128,18 +131,32 @@ dkv_status finish_plan(dkv_plan* p)
 {
     cudaGetDevice(&p->device);
     p->use_mma = p->total_rows >= 1 && p->total_rows <= dkv::kMaxMmaRows;
-    cudaError_t e = p->use_mma ? dkv::decode_config_mma(p->G, p->B, &p->cfg) : dkv::decode_config(p->G, p->B, &p->cfg);
-    if (e != cudaSuccess) return cuda_fail(e, "decode_config");
-    p->slots = (int64_t)p->cfg.nctas + p->B * p->s.H_kv;
-    dkv_status st = dalloc(&p->d_work, (size_t)dkv::decode_workspace_floats(p->cfg, p->G, p->B * p->s.H_kv),
+    cudaError_t e;
+    if (p->use_mma) {
+        if ((e = dkv::decode_config_mma(p->G, p->B, 1, &p->cfg)) != cudaSuccess) return cuda_fail(e, "decode_config");
+        if ((e = dkv::decode_config_mma(p->G, p->B, 2, &p->cfg_multi)) != cudaSuccess)
+            return cuda_fail(e, "decode_config (multi-query)");
+        p->nctas_cap = std::max(p->cfg.nctas, p->cfg_multi.nctas);
+        p->warps_cap = std::max(p->cfg.nwarps, p->cfg_multi.nwarps);
+        p->cols_cap = dkv::kMaxCols;
+    } else {
+        if ((e = dkv::decode_config(p->G, p->B, &p->cfg)) != cudaSuccess) return cuda_fail(e, "decode_config");
+        p->nctas_cap = p->cfg.nctas;
+        p->warps_cap = p->cfg.nwarps;
+        p->cols_cap = p->G;
+    }
+    p->slots = (int64_t)p->nctas_cap + p->B * p->s.H_kv;
+    dkv_status st = dalloc(&p->d_work,
+                           (size_t)dkv::decode_workspace_floats(p->nctas_cap, p->warps_cap, p->cols_cap,
+                                                                p->B * p->s.H_kv),
                            "split-K workspace");
     if (st != DKV_OK) return st;
     st = dalloc(&p->d_status, 1, "status word");
     if (st != DKV_OK) return st;
     if ((e = cudaMemset(p->d_status, 0, sizeof(int32_t))) != cudaSuccess) return cuda_fail(e, "cudaMemset");
-    st = dalloc(&p->d_slab_count, (size_t)p->B * p->s.H_kv * p->G, "slab counters");
+    st = dalloc(&p->d_slab_count, (size_t)p->B * p->s.H_kv * p->cols_cap, "slab counters");
     if (st != DKV_OK) return st;
-    if ((e = cudaMemset(p->d_slab_count, 0, sizeof(int32_t) * p->B * p->s.H_kv * p->G)) != cudaSuccess)
+    if ((e = cudaMemset(p->d_slab_count, 0, sizeof(int32_t) * p->B * p->s.H_kv * p->cols_cap)) != cudaSuccess)
         return cuda_fail(e, "cudaMemset");
     return DKV_OK;
 }
@@ -439,11 +456,11 @@ dkv_status decode_args(const dkv_plan* p, int32_t layer, const void* q, const vo
     a->len = p->d_len + (int64_t)layer * NHl;
     a->off = p->d_off + (int64_t)layer * NHl;
     a->ioff = p->d_ioff + (int64_t)layer * NHl;
-    const size_t nw = (size_t)p->cfg.nctas * p->cfg.nwarps;
+    const size_t nw = (size_t)p->nctas_cap * p->warps_cap;
     a->work_o = p->d_work;
-    a->work_ml = a->work_o + (size_t)p->slots * p->G * dkv::kHeadDim;
-    a->warp_o = a->work_ml + (size_t)p->slots * p->G * 2;
-    a->warp_ml = a->warp_o + nw * p->G * dkv::kHeadDim;
+    a->work_ml = a->work_o + (size_t)p->slots * p->cols_cap * dkv::kHeadDim;
+    a->warp_o = a->work_ml + (size_t)p->slots * p->cols_cap * 2;
+    a->warp_ml = a->warp_o + nw * p->cols_cap * dkv::kHeadDim;
     a->out = out;
     a->slab_count = p->d_slab_count;
     a->status = p->d_status;
@@ -451,6 +468,8 @@ dkv_status decode_args(const dkv_plan* p, int32_t layer, const void* q, const vo
     a->H = p->s.H;
     a->Hkv = p->s.H_kv;
     a->G = p->G;
+    a->Q = 1;
+    a->NC = p->G;
     a->reserve = p->reserve;
     a->append = with_new ? 1 : 0;
     const float sc = scale > 0.f ? scale : 1.0f / std::sqrt((float)dkv::kHeadDim);
@@ -486,6 +505,29 @@ dkv_status dkv_decode_attn(const dkv_plan* p, int32_t layer, const void* q, cons
                                 true, true, &a);
     if (st != DKV_OK) return st;
     st = launch_split_k(p, a, true, stream);
+    return st == DKV_OK ? ok() : st;
+}
+
+dkv_status dkv_decode_multi(const dkv_plan* p, int32_t layer, const void* q, int32_t num_queries,
+                            const int32_t* n_appended, void* Kc, void* Vc, float scale, float* out,
+                            cudaStream_t stream)
+{
+    dkv::DecodeArgs a;
+    dkv_status st = decode_args(p, layer, q, nullptr, nullptr, 0, n_appended, Kc, Vc, scale, out, true, true, &a);
+    if (st != DKV_OK) return st;
+    if (num_queries < 1 || num_queries * p->G > dkv::kMaxCols)
+        return fail(DKV_ERR_INVALID_ARG, "num_queries=%d: need 1 <= Q and Q*G <= %d (G=%d)", num_queries,
+                    dkv::kMaxCols, p->G);
+    if (!p->use_mma)
+        return fail(DKV_ERR_INVALID_ARG, "multi-query decode needs the tensor-core kernel (a cache of < 2^31 rows)");
+    a.Q = num_queries;
+    a.NC = num_queries * p->G;
+    const dkv::DecodeConfig& cfg = a.NC > 8 ? p->cfg_multi : p->cfg;
+    a.nctas = cfg.nctas;
+    dkv::CacheMaps maps;
+    const cudaError_t e = dkv::make_cache_maps(a.Kc, a.Vc, p->total_rows, &maps);
+    if (e != cudaSuccess) return cuda_fail(e, "tensor maps of the packed caches");
+    st = launched(dkv::launch_decode_mma_fused(a, maps, cfg, stream), "multi-query decode kernel");
     return st == DKV_OK ? ok() : st;
 }
 

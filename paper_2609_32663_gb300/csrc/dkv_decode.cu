@@ -541,7 +541,7 @@ __global__ void __launch_bounds__(C::NW * 32, 1) decode_partial_kernel(const Dec
     __syncthreads();
     pdl_wait();  // the merges write the workspace and out: the previous kernel must be done with them
 
-    cta_tail<G, NW, FUSED>(a, smem, NS * C::kStageBytes, seg_first, c, R, warp, lane);
+    cta_tail<G, NW, FUSED, G>(a, smem, NS * C::kStageBytes, seg_first, c, R, warp, lane);
 }
 
 // ------------------------------------------------------------ combine kernel

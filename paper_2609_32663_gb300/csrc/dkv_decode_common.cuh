@@ -237,12 +237,20 @@ __device__ __forceinline__ int ctas_of_slab(int p0, int p1, int R, int P, int* c
     return n;
 }
 
-// out[b][g*G + j] = O / L for the group's heads; O, L per head j for the lane's 4 dims.
+// Output row of column c of slab (b, g): query c / G, head g G + c % G of out [B][Q][H][128].
 template <int G>
-__device__ __forceinline__ void write_out(const DecodeArgs& a, int b, int g, int j, float4 O, float L, int lane)
+__device__ __forceinline__ int64_t out_row(const DecodeArgs& a, int b, int g, int c)
+{
+    const int qi = c / G, j = c - qi * G;
+    return ((int64_t)b * a.Q + qi) * a.H + g * G + j;
+}
+
+// out row of column c = O / L; O, L of the column for the lane's 4 dims.
+template <int G>
+__device__ __forceinline__ void write_out(const DecodeArgs& a, int b, int g, int c, float4 O, float L, int lane)
 {
     const float inv = L > 0.f ? 1.f / L : 0.f;
-    float4* dst = reinterpret_cast<float4*>(a.out + ((int64_t)b * a.H + g * G + j) * kHeadDim);
+    float4* dst = reinterpret_cast<float4*>(a.out + out_row<G>(a, b, g, c) * kHeadDim);
     dst[lane] = make_float4(O.x * inv, O.y * inv, O.z * inv, O.w * inv);
 }
 
@@ -253,7 +261,7 @@ __device__ __forceinline__ void write_out(const DecodeArgs& a, int b, int g, int
 // load round at the end of a launch takes ~1.5 us and grows with the bytes in
 // flight, so one round of 20-24 partials costs more than two smaller ones; of
 // 8, 10, 12, 16, 20 and 24, KB = 12 was fastest.
-template <int G, int KB>
+template <int G, int KB, int NCC>
 __device__ void merge_slab_head(const DecodeArgs& a, int h, int j, int c0, int c1, int R, int lane)
 {
     const int b = h / a.Hkv, g = h - b * a.Hkv;
@@ -268,7 +276,7 @@ __device__ void merge_slab_head(const DecodeArgs& a, int h, int j, int c0, int c
         for (int u = 0; u < KB; ++u) {
             const int cc = k0 + u;
             const bool ok = cc <= c1 && (all_live || part_start(cc, R, P) < part_start(cc + 1, R, P));
-            const int64_t sj = ((int64_t)cc + h) * G + j;
+            const int64_t sj = ((int64_t)cc + h) * (NCC ? NCC : a.NC) + j;
             ml[u] = ok ? __ldcg(reinterpret_cast<const float2*>(a.work_ml + sj * 2)) : make_float2(-INFINITY, 0.f);
             v[u] = ok ? __ldcg(reinterpret_cast<const float4*>(a.work_o + sj * kHeadDim) + lane)
                       : make_float4(0.f, 0.f, 0.f, 0.f);
@@ -297,7 +305,8 @@ __device__ void merge_slab_head(const DecodeArgs& a, int h, int j, int c0, int c
 }
 
 // End of one CTA's split-K pass, after its warps' ranges are done and a CTA
-// barrier. meta: seg_first[NW], seg_last[NW] (first / last slab of warp w, -1 if
+// barrier. NCC: the number of columns per slab when fixed at compile time (the
+// decode step: G), 0 to take a.NC. meta: seg_first[NW], seg_last[NW] (first / last slab of warp w, -1 if
 // none), then the layer rows [p0, p1) of each entry (2 w: first, 2 w + 1: last)
 // as p0[2 NW], p1[2 NW], recorded while streaming so the end of the pass reads
 // no plan metadata from global memory;
@@ -307,7 +316,7 @@ __device__ void merge_slab_head(const DecodeArgs& a, int h, int j, int c0, int c
 // is written out (fused), otherwise the CTA writes its partial to slot c + h
 // and, fused, counts itself in for each (slab, head): the last CTA to arrive
 // merges all CTA partials of that (slab, head).
-template <int G, int NW, bool FUSED>
+template <int G, int NW, bool FUSED, int NCC>
 __device__ void cta_tail(const DecodeArgs& a, const unsigned char* ring, int warp_ring_bytes,
                          const int32_t* meta, int c, int R, int warp, int lane)
 {
@@ -329,8 +338,16 @@ __device__ void cta_tail(const DecodeArgs& a, const unsigned char* ring, int war
     }
     const unsigned fresh = __ballot_sync(kFull, h_e >= 0 && h_e != prev);
     const int nslab = __popc(fresh);
-    for (int t = warp; t < nslab * G; t += NW) {
-        const int si = t / G, j = t - si * G;
+    const int NC = NCC ? NCC : a.NC;  // columns (query x head) per slab; NCC: known at compile time
+    // Task t = (slab #si, column j), t = si NC + j; warp w takes t = w, w + NW, ...
+    // (si, j) advance by additions: no division on this latency-bound path.
+    int si = 0, j = warp - NW;
+    for (int t = warp; t < nslab * NC; t += NW) {
+        j += NW;
+        while (j >= NC) {
+            j -= NC;
+            ++si;
+        }
         unsigned m = fresh;
         for (int k = 0; k < si; ++k) m &= m - 1;
         const int e0 = __ffs(m) - 1;
@@ -344,8 +361,8 @@ __device__ void cta_tail(const DecodeArgs& a, const unsigned char* ring, int war
         for (int f = 0; f < 2 * NW; ++f) {
             if (!((same >> f) & 1u)) continue;
             const int w = f >> 1;
-            const float* ml = (f & 1) ? reinterpret_cast<const float*>(ring + w * warp_ring_bytes) + G * kHeadDim
-                                      : a.warp_ml + ((int64_t)c * NW + w) * G * 2;
+            const float* ml = (f & 1) ? reinterpret_cast<const float*>(ring + w * warp_ring_bytes) + NC * kHeadDim
+                                      : a.warp_ml + ((int64_t)c * NW + w) * NC * 2;
             M = fmaxf(M, ml[2 * j]);
         }
         float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -355,8 +372,8 @@ __device__ void cta_tail(const DecodeArgs& a, const unsigned char* ring, int war
             if (!((same >> f) & 1u)) continue;
             const int w = f >> 1;
             const float* ob = (f & 1) ? reinterpret_cast<const float*>(ring + w * warp_ring_bytes)
-                                      : a.warp_o + ((int64_t)c * NW + w) * G * kHeadDim;
-            const float* ml = (f & 1) ? ob + G * kHeadDim : a.warp_ml + ((int64_t)c * NW + w) * G * 2;
+                                      : a.warp_o + ((int64_t)c * NW + w) * NC * kHeadDim;
+            const float* ml = (f & 1) ? ob + NC * kHeadDim : a.warp_ml + ((int64_t)c * NW + w) * NC * 2;
             const float2 mlj = *reinterpret_cast<const float2*>(ml + 2 * j);
             const float fct = (mlj.x == -INFINITY) ? 0.f : ex2(mlj.x - M);
             L = fmaf(mlj.y, fct, L);
@@ -371,15 +388,15 @@ __device__ void cta_tail(const DecodeArgs& a, const unsigned char* ring, int war
             continue;
         }
         const int64_t slot = (int64_t)c + h;
-        reinterpret_cast<float4*>(a.work_o + (slot * G + j) * kHeadDim)[lane] = O;
-        if (lane == 0) *reinterpret_cast<float2*>(a.work_ml + (slot * G + j) * 2) = make_float2(M, L);
+        reinterpret_cast<float4*>(a.work_o + (slot * NC + j) * kHeadDim)[lane] = O;
+        if (lane == 0) *reinterpret_cast<float2*>(a.work_ml + (slot * NC + j) * 2) = make_float2(M, L);
         if (!FUSED) continue;
         // Count this CTA in for (slab, head): release of the partial just written,
         // and, for the last CTA, acquire of the others' before merging them.
         __syncwarp();
         int last = 0;
         if (lane == 0) {
-            int32_t* ctr = a.slab_count + (int64_t)h * G + j;
+            int32_t* ctr = a.slab_count + (int64_t)h * NC + j;
             int old;
             asm volatile("atom.add.acq_rel.gpu.s32 %0, [%1], 1;" : "=r"(old) : "l"(ctr) : "memory");
             last = (old == nct - 1) ? 1 : 0;
@@ -387,7 +404,7 @@ __device__ void cta_tail(const DecodeArgs& a, const unsigned char* ring, int war
         }
         last = __shfl_sync(kFull, last, 0);
         __syncwarp();
-        if (last) merge_slab_head<G, 12>(a, h, j, c0h, c1h, R, lane);
+        if (last) merge_slab_head<G, 12, NCC>(a, h, j, c0h, c1h, R, lane);
     }
 }
 

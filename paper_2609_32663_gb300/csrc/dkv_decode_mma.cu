@@ -35,9 +35,9 @@ constexpr int kMmaTR = 16;                // rows per tile: the m16 of the score
 constexpr int kBoxBytes = kMmaTR * 128;   // one TMA box: 16 rows x 64 bf16 dims
 constexpr int kMmaStage = 4 * kBoxBytes;  // K dims 0-63, K dims 64-127, V dims 0-63, V dims 64-127
 
-template <int G_, int NS_, int NW_>
+template <int G_, int NT_, int NS_, int NW_>
 struct MK {
-    static constexpr int G = G_, NS = NS_, NW = NW_, TR = kMmaTR;
+    static constexpr int G = G_, NT = NT_, NS = NS_, NW = NW_, TR = kMmaTR;
     static constexpr int kStageBytes = kMmaStage;
     static constexpr int kWarpRing = NS * kStageBytes;
     static constexpr int kRingBytes = NW * kWarpRing;
@@ -46,21 +46,28 @@ struct MK {
     static constexpr int kAlign = 1024;                  // swizzle atoms are 1024-byte aligned
     static constexpr int kFixedBytes = kRingBytes + kBarBytes + kMetaBytes;
     static int bytes(int B) { return kAlign + kFixedBytes + (2 * B + 1) * 4; }
-    static_assert(G * (kHeadDim + 2) * 4 <= kWarpRing, "a warp's final state fits in its ring");
+    static_assert(8 * NT * (kHeadDim + 2) * 4 <= kWarpRing, "a warp's final state fits in its ring");
 };
 
-// Stages per warp, warps per CTA. The ring holds 192 KB per SM either way; more
-// warps hide more of a tile's latency chain (8 dependent score MMAs, softmax,
-// 16 output MMAs), and at the end of a pass the CTA's (slab, head) merge tasks
-// spread over more warps, which counts for G > 4 (G tasks per slab).
+// Stages per warp, warps per CTA. One column tile (the decode step): more warps
+// hide more of a tile's latency chain (8 dependent score MMAs, softmax, 16
+// output MMAs), and at the end of a pass the CTA's (slab, column) merge tasks
+// spread over more warps, which counts for G > 4 (G tasks per slab). Two column
+// tiles (multi-query): twice the accumulators, so 8 warps with the full
+// register file, and stages enough to hold a 16-column final state.
 #ifndef DKV_MMA_CFG_SMALL_G
 #define DKV_MMA_CFG_SMALL_G 2, 12
 #endif
 #ifndef DKV_MMA_CFG_LARGE_G
 #define DKV_MMA_CFG_LARGE_G 1, 16
 #endif
-template <int G>
-using MKFor = typename std::conditional<(G <= 4), MK<G, DKV_MMA_CFG_SMALL_G>, MK<G, DKV_MMA_CFG_LARGE_G>>::type;
+#ifndef DKV_MMA_CFG_MULTI
+#define DKV_MMA_CFG_MULTI 3, 8
+#endif
+template <int G, int NT>
+using MKFor = typename std::conditional<
+    (NT > 1), MK<G, NT, DKV_MMA_CFG_MULTI>,
+    typename std::conditional<(G <= 4), MK<G, 1, DKV_MMA_CFG_SMALL_G>, MK<G, 1, DKV_MMA_CFG_LARGE_G>>::type>::type;
 
 // ------------------------------------------------------------ PTX wrappers
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar,
@@ -116,167 +123,217 @@ __device__ __forceinline__ uint32_t bf16x2(float lo, float hi)
 __device__ __forceinline__ int swz(int r, int ch) { return r * 128 + ((ch ^ (r & 7)) << 4); }
 
 // ------------------------------------------------------------ per-warp state
-// Lane (gid = lane / 4, t = lane % 4) holds heads 2t and 2t+1 of the group.
+// Columns: the n side of both products, NT tiles of 8. Column c is query c / G,
+// head c % G of the KV head's group (the decode step has one query: c = head).
+// Lane (gid = lane / 4, t = lane % 4) holds columns 8 nt + 2t and 8 nt + 2t + 1.
+template <int NT>
 struct MmaState {
-    float m[2];     // running max of the two heads (log2 domain), the same in all gid lanes
-    float l[2];     // this lane's share of their softmax denominators
-    float o[8][4];  // O^T: [dim block db][(dim 16 db + gid, head 2t), (.., 2t+1), (dim +8, 2t), (dim +8, 2t+1)]
+    float m[NT][2];     // running max of the two columns (log2 domain), the same in all gid lanes
+    float l[NT][2];     // this lane's share of their softmax denominators
+    float o[NT][8][4];  // O^T: [tile][dim block db][(dim 16 db + gid, col 2t), (.., 2t+1), (dim +8, 2t), (.., 2t+1)]
 };
 
-__device__ __forceinline__ void state_reset(MmaState& S)
+template <int NT>
+__device__ __forceinline__ void state_reset(MmaState<NT>& S)
 {
-    S.m[0] = S.m[1] = -INFINITY;
-    S.l[0] = S.l[1] = 0.f;
 #pragma unroll
-    for (int db = 0; db < 8; ++db) S.o[db][0] = S.o[db][1] = S.o[db][2] = S.o[db][3] = 0.f;
+    for (int nt = 0; nt < NT; ++nt) {
+        S.m[nt][0] = S.m[nt][1] = -INFINITY;
+        S.l[nt][0] = S.l[nt][1] = 0.f;
+#pragma unroll
+        for (int db = 0; db < 8; ++db) S.o[nt][db][0] = S.o[nt][db][1] = S.o[nt][db][2] = S.o[nt][db][3] = 0.f;
+    }
 }
 
-// q of the group as B fragments of the score product: for k step kk (dims
-// 16 kk .. 16 kk + 15), (head gid, dims 2t, 2t+1) and (head gid, dims 2t+8, 2t+9).
-template <int G>
-__device__ __forceinline__ void load_q(const DecodeArgs& a, int b, int g, int lane, uint32_t (&qb)[8][2])
+// q of the slab's columns as B fragments of the score product: for tile nt and k
+// step kk (dims 16 kk .. 16 kk + 15), (column 8 nt + gid, dims 2t, 2t+1) and
+// (column 8 nt + gid, dims 2t+8, 2t+9); zero past the last column.
+template <int G, int NT>
+__device__ __forceinline__ void load_q(const DecodeArgs& a, int b, int g, int NC, int lane, uint32_t (&qb)[NT][8][2])
 {
     const int gid = lane >> 2, t = lane & 3;
-    const bool live = gid < G;
-    const uint32_t* qr = reinterpret_cast<const uint32_t*>(a.q + ((int64_t)b * a.H + g * G + (live ? gid : 0)) * kHeadDim);
 #pragma unroll
-    for (int kk = 0; kk < 8; ++kk) {
-        qb[kk][0] = live ? __ldg(qr + 8 * kk + t) : 0u;
-        qb[kk][1] = live ? __ldg(qr + 8 * kk + t + 4) : 0u;
+    for (int nt = 0; nt < NT; ++nt) {
+        const int col = 8 * nt + gid;
+        const bool live = col < NC;
+        const int qi = col / G, j = col - qi * G;
+        const uint32_t* qr =
+            reinterpret_cast<const uint32_t*>(a.q + (live ? ((int64_t)b * a.Q + qi) * a.H + g * G + j : 0) * kHeadDim);
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+            qb[nt][kk][0] = live ? __ldg(qr + 8 * kk + t) : 0u;
+            qb[nt][kk][1] = live ? __ldg(qr + 8 * kk + t + 4) : 0u;
+        }
     }
 }
 
 // One tile: stage holds K (boxes 0, 1) and V (boxes 2, 3); rows >= cnt are not
 // part of the segment (their V rows must already be zero when !FULL).
-template <bool FULL>
-__device__ __forceinline__ void mma_tile(MmaState& S, const uint32_t (&qb)[8][2], uint32_t stage, int cnt, float cs,
-                                         int lane)
+template <bool FULL, int NT>
+__device__ __forceinline__ void mma_tile(MmaState<NT>& S, const uint32_t (&qb)[NT][8][2], uint32_t stage, int cnt,
+                                         float cs, int lane)
 {
     const int gid = lane >> 2;
     // Scores: ldmatrix lane -> (row, chunk) of the A fragment: rows 0-7 / 8-15 by
-    // bit 3 of the lane, chunk +0 / +1 by bit 4.
+    // bit 3 of the lane, chunk +0 / +1 by bit 4. One K fragment serves all tiles.
     const int ar = (lane & 7) + (lane & 8), ac = lane >> 4;
-    float c[4] = {0.f, 0.f, 0.f, 0.f};
+    float c[NT][4];
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) c[nt][0] = c[nt][1] = c[nt][2] = c[nt][3] = 0.f;
 #pragma unroll
     for (int kk = 0; kk < 8; ++kk) {
         uint32_t af[4];
         ldsm_x4(stage + (kk >> 2) * kBoxBytes + swz(ar, (kk & 3) * 2 + ac), af);
-        mma16816(c, af, qb[kk][0], qb[kk][1]);
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) mma16816(c[nt], af, qb[nt][kk][0], qb[nt][kk][1]);
     }
-    // c: (row gid, heads 2t, 2t+1), (row gid + 8, heads 2t, 2t+1).
-    float s0 = c[0] * cs, s1 = c[1] * cs, s2 = c[2] * cs, s3 = c[3] * cs;
-    if (!FULL) {
-        if (gid >= cnt) s0 = s1 = -INFINITY;
-        if (gid + 8 >= cnt) s2 = s3 = -INFINITY;
-    }
-    // Lazy rescaling as in the fp32 kernel: the running max only moves when a
+    uint32_t bh0[NT], bh1[NT], bl0[NT], bl1[NT];
+    // c: (row gid, columns 2t, 2t+1), (row gid + 8, columns 2t, 2t+1). Lazy
+    // rescaling as in the fp32 kernel: a column's running max only moves when a
     // score tops it by more than kSlack.
-    const float x0 = fmaxf(s0, s2), x1 = fmaxf(s1, s3);
-    if (__any_sync(kFull, x0 > S.m[0] + kSlack || x1 > S.m[1] + kSlack)) {
-        float y0 = x0, y1 = x1;
+    float s[NT][4];
+    bool over = false;
 #pragma unroll
-        for (int o = 4; o <= 16; o <<= 1) {
-            y0 = fmaxf(y0, __shfl_xor_sync(kFull, y0, o));
-            y1 = fmaxf(y1, __shfl_xor_sync(kFull, y1, o));
-        }
-        const float mn0 = fmaxf(S.m[0], y0), mn1 = fmaxf(S.m[1], y1);
-        const float al0 = (mn0 == -INFINITY) ? 1.f : ex2(S.m[0] - mn0);
-        const float al1 = (mn1 == -INFINITY) ? 1.f : ex2(S.m[1] - mn1);
-        S.l[0] *= al0;
-        S.l[1] *= al1;
+    for (int nt = 0; nt < NT; ++nt) {
 #pragma unroll
-        for (int db = 0; db < 8; ++db) {
-            S.o[db][0] *= al0;
-            S.o[db][1] *= al1;
-            S.o[db][2] *= al0;
-            S.o[db][3] *= al1;
+        for (int i = 0; i < 4; ++i) s[nt][i] = c[nt][i] * cs;
+        if (!FULL) {
+            if (gid >= cnt) s[nt][0] = s[nt][1] = -INFINITY;
+            if (gid + 8 >= cnt) s[nt][2] = s[nt][3] = -INFINITY;
         }
-        S.m[0] = mn0;
-        S.m[1] = mn1;
+        over |= fmaxf(s[nt][0], s[nt][2]) > S.m[nt][0] + kSlack || fmaxf(s[nt][1], s[nt][3]) > S.m[nt][1] + kSlack;
     }
-    const float r0 = (S.m[0] == -INFINITY) ? 0.f : S.m[0], r1 = (S.m[1] == -INFINITY) ? 0.f : S.m[1];
-    const float p0 = ex2(s0 - r0), p1 = ex2(s1 - r1), p2 = ex2(s2 - r0), p3 = ex2(s3 - r1);  // 2^-inf = 0
-    S.l[0] += p0 + p2;
-    S.l[1] += p1 + p3;
-    // P^T as B fragments: bf16 high part and remainder, transposed by movmatrix
-    // from (row, head pair) to (row pair, head).
-    const uint32_t h01 = bf16x2(p0, p1), h23 = bf16x2(p2, p3);
-    const uint32_t l01 = bf16x2(p0 - __uint_as_float(h01 << 16), p1 - __uint_as_float(h01 & 0xffff0000u));
-    const uint32_t l23 = bf16x2(p2 - __uint_as_float(h23 << 16), p3 - __uint_as_float(h23 & 0xffff0000u));
-    const uint32_t bh0 = movm_t(h01), bh1 = movm_t(h23), bl0 = movm_t(l01), bl1 = movm_t(l23);
+    if (__any_sync(kFull, over)) {
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+            float y0 = fmaxf(s[nt][0], s[nt][2]), y1 = fmaxf(s[nt][1], s[nt][3]);
+#pragma unroll
+            for (int o = 4; o <= 16; o <<= 1) {
+                y0 = fmaxf(y0, __shfl_xor_sync(kFull, y0, o));
+                y1 = fmaxf(y1, __shfl_xor_sync(kFull, y1, o));
+            }
+            const float mn0 = fmaxf(S.m[nt][0], y0), mn1 = fmaxf(S.m[nt][1], y1);
+            const float al0 = (mn0 == -INFINITY) ? 1.f : ex2(S.m[nt][0] - mn0);
+            const float al1 = (mn1 == -INFINITY) ? 1.f : ex2(S.m[nt][1] - mn1);
+            S.l[nt][0] *= al0;
+            S.l[nt][1] *= al1;
+#pragma unroll
+            for (int db = 0; db < 8; ++db) {
+                S.o[nt][db][0] *= al0;
+                S.o[nt][db][1] *= al1;
+                S.o[nt][db][2] *= al0;
+                S.o[nt][db][3] *= al1;
+            }
+            S.m[nt][0] = mn0;
+            S.m[nt][1] = mn1;
+        }
+    }
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+        const float r0 = (S.m[nt][0] == -INFINITY) ? 0.f : S.m[nt][0];
+        const float r1 = (S.m[nt][1] == -INFINITY) ? 0.f : S.m[nt][1];
+        const float p0 = ex2(s[nt][0] - r0), p1 = ex2(s[nt][1] - r1);  // 2^-inf = 0
+        const float p2 = ex2(s[nt][2] - r0), p3 = ex2(s[nt][3] - r1);
+        S.l[nt][0] += p0 + p2;
+        S.l[nt][1] += p1 + p3;
+        // P^T as B fragments: bf16 high part and remainder, transposed by movmatrix
+        // from (row, column pair) to (row pair, column).
+        const uint32_t h01 = bf16x2(p0, p1), h23 = bf16x2(p2, p3);
+        const uint32_t l01 = bf16x2(p0 - __uint_as_float(h01 << 16), p1 - __uint_as_float(h01 & 0xffff0000u));
+        const uint32_t l23 = bf16x2(p2 - __uint_as_float(h23 << 16), p3 - __uint_as_float(h23 & 0xffff0000u));
+        bh0[nt] = movm_t(h01);
+        bh1[nt] = movm_t(h23);
+        bl0[nt] = movm_t(l01);
+        bl1[nt] = movm_t(l23);
+    }
     // O^T += V^T P^T: ldmatrix.trans lane -> (row, chunk): rows 0-7 / 8-15 by
-    // bit 4 of the lane, chunk +0 / +1 by bit 3.
+    // bit 4 of the lane, chunk +0 / +1 by bit 3. One V fragment serves all tiles.
     const int vr = (lane & 7) + ((lane >> 4) << 3), vc = (lane >> 3) & 1;
     const uint32_t vt = stage + 2 * kBoxBytes;
 #pragma unroll
     for (int db = 0; db < 8; ++db) {
         uint32_t af[4];
         ldsm_x4_t(vt + (db >> 2) * kBoxBytes + swz(vr, (db & 3) * 2 + vc), af);
-        mma16816(S.o[db], af, bh0, bh1);
-        mma16816(S.o[db], af, bl0, bl1);
-    }
-}
-
-// Softmax denominators of the lane's two heads, summed over the gid lanes.
-__device__ __forceinline__ void finish_l(const MmaState& S, float (&l2)[2])
-{
-    float a = S.l[0], b = S.l[1];
 #pragma unroll
-    for (int o = 4; o <= 16; o <<= 1) {
-        a += __shfl_xor_sync(kFull, a, o);
-        b += __shfl_xor_sync(kFull, b, o);
-    }
-    l2[0] = a;
-    l2[1] = b;
-}
-
-// The state as a record: o[G][128] at o_dst, (m, l)[G] at ml_dst (heads < G).
-template <int G>
-__device__ __forceinline__ void store_mma_state(const MmaState& S, const float (&l2)[2], float* o_dst, float* ml_dst,
-                                                int lane)
-{
-    const int gid = lane >> 2, t = lane & 3;
-#pragma unroll
-    for (int q = 0; q < 2; ++q) {
-        const int j = 2 * t + q;
-        if (j < G) {
-#pragma unroll
-            for (int db = 0; db < 8; ++db) {
-                o_dst[j * kHeadDim + 16 * db + gid] = S.o[db][q];
-                o_dst[j * kHeadDim + 16 * db + gid + 8] = S.o[db][2 + q];
-            }
-            if (gid == 0) *reinterpret_cast<float2*>(ml_dst + 2 * j) = make_float2(S.m[q], l2[q]);
+        for (int nt = 0; nt < NT; ++nt) {
+            mma16816(S.o[nt][db], af, bh0[nt], bh1[nt]);
+            mma16816(S.o[nt][db], af, bl0[nt], bl1[nt]);
         }
     }
 }
 
-// Final answer of a slab held by one warp: out = o / l.
-template <int G>
-__device__ __forceinline__ void write_mma_out(const DecodeArgs& a, const MmaState& S, const float (&l2)[2], int b,
-                                              int g, int lane)
+// Softmax denominators of the lane's columns, summed over the gid lanes.
+template <int NT>
+__device__ __forceinline__ void finish_l(const MmaState<NT>& S, float (&l2)[NT][2])
+{
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+        float a = S.l[nt][0], b = S.l[nt][1];
+#pragma unroll
+        for (int o = 4; o <= 16; o <<= 1) {
+            a += __shfl_xor_sync(kFull, a, o);
+            b += __shfl_xor_sync(kFull, b, o);
+        }
+        l2[nt][0] = a;
+        l2[nt][1] = b;
+    }
+}
+
+// The state as a record: o[NC][128] at o_dst, (m, l)[NC] at ml_dst.
+template <int NT>
+__device__ __forceinline__ void store_mma_state(const MmaState<NT>& S, const float (&l2)[NT][2], float* o_dst,
+                                                float* ml_dst, int NC, int lane)
 {
     const int gid = lane >> 2, t = lane & 3;
 #pragma unroll
-    for (int q = 0; q < 2; ++q) {
-        const int j = 2 * t + q;
-        if (j < G) {
-            const float inv = l2[q] > 0.f ? 1.f / l2[q] : 0.f;
-            float* dst = a.out + ((int64_t)b * a.H + g * G + j) * kHeadDim;
+    for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
-            for (int db = 0; db < 8; ++db) {
-                dst[16 * db + gid] = S.o[db][q] * inv;
-                dst[16 * db + gid + 8] = S.o[db][2 + q] * inv;
+        for (int q = 0; q < 2; ++q) {
+            const int j = 8 * nt + 2 * t + q;
+            if (j < NC) {
+#pragma unroll
+                for (int db = 0; db < 8; ++db) {
+                    o_dst[j * kHeadDim + 16 * db + gid] = S.o[nt][db][q];
+                    o_dst[j * kHeadDim + 16 * db + gid + 8] = S.o[nt][db][2 + q];
+                }
+                if (gid == 0) *reinterpret_cast<float2*>(ml_dst + 2 * j) = make_float2(S.m[nt][q], l2[nt][q]);
             }
         }
-    }
+}
+
+// Final answer of a slab held by one warp: out = o / l for every column.
+template <int G, int NT>
+__device__ __forceinline__ void write_mma_out(const DecodeArgs& a, const MmaState<NT>& S, const float (&l2)[NT][2],
+                                              int b, int g, int NC, int lane)
+{
+    const int gid = lane >> 2, t = lane & 3;
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+            const int j = 8 * nt + 2 * t + q;
+            if (j < NC) {
+                const float inv = l2[nt][q] > 0.f ? 1.f / l2[nt][q] : 0.f;
+                float* dst = a.out + out_row<G>(a, b, g, j) * kHeadDim;
+#pragma unroll
+                for (int db = 0; db < 8; ++db) {
+                    dst[16 * db + gid] = S.o[nt][db][q] * inv;
+                    dst[16 * db + gid + 8] = S.o[nt][db][2 + q] * inv;
+                }
+            }
+        }
 }
 
 // ------------------------------------------------------------ kernel
-template <int G, bool FUSED>
-__global__ void __launch_bounds__(MKFor<G>::NW * 32, 1)
+// MULTI: columns are Q x G with Q from the arguments (multi-query); otherwise
+// the G heads of the decode step, fixed at compile time.
+template <int G, int NT, bool FUSED, bool MULTI>
+__global__ void __launch_bounds__(MKFor<G, NT>::NW * 32, 1)
     decode_mma_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ CacheMaps maps)
 {
-    using C = MKFor<G>;
+    using C = MKFor<G, NT>;
+    constexpr int NCC = MULTI ? 0 : G;
+    const int NC = MULTI ? a.NC : G;
     constexpr int TR = C::TR, NS = C::NS, NW = C::NW;
     extern __shared__ __align__(128) unsigned char smem_raw[];
     // The ring starts on a 1024-byte boundary (the swizzle pattern's period).
@@ -311,7 +368,7 @@ __global__ void __launch_bounds__(MKFor<G>::NW * 32, 1)
         pdl_wait();
         for (int h = 0; h < NHl; ++h)
             if (slab_start(a, tab, h) == slab_start(a, tab, h + 1))
-                for (int j = 0; j < G; ++j)
+                for (int j = 0; j < NC; ++j)
                     write_out<G>(a, h / a.Hkv, h % a.Hkv, j, make_float4(0.f, 0.f, 0.f, 0.f), 0.f, lane);
     }
     const int A = part_start(c, R, a.nctas), Bc = part_start(c + 1, R, a.nctas);
@@ -319,8 +376,8 @@ __global__ void __launch_bounds__(MKFor<G>::NW * 32, 1)
     const int wA = A + (int)(((int64_t)(Bc - A) * warp) / NW);
     const int wB = A + (int)(((int64_t)(Bc - A) * (warp + 1)) / NW);
     unsigned char* my_ring = smem + warp * C::kWarpRing;
-    MmaState S;
-    float l2[2];
+    MmaState<NT> S;
+    float l2[NT][2];
     bool have_last = false;  // S holds the state of this warp's last slab
 
     if (wA < wB) {
@@ -387,8 +444,8 @@ __global__ void __launch_bounds__(MKFor<G>::NW * 32, 1)
             const int h = cp.h;
             const int p0h = cp.p0, p1h = cp.p0 + cp.n_h;  // the slab's layer rows
             const int b = h / a.Hkv, g = h - b * a.Hkv;
-            uint32_t qb[8][2];
-            load_q<G>(a, b, g, lane, qb);
+            uint32_t qb[NT][8][2];
+            load_q<G, NT>(a, b, g, NC, lane, qb);
             state_reset(S);
 
             while (cp.h == h) {
@@ -429,9 +486,9 @@ __global__ void __launch_bounds__(MKFor<G>::NW * 32, 1)
                     __syncwarp();
                 }
                 if (cnt == TR)
-                    mma_tile<true>(S, qb, smem_u32(st), cnt, cs, lane);
+                    mma_tile<true, NT>(S, qb, smem_u32(st), cnt, cs, lane);
                 else
-                    mma_tile<false>(S, qb, smem_u32(st), cnt, cs, lane);
+                    mma_tile<false, NT>(S, qb, smem_u32(st), cnt, cs, lane);
                 __syncwarp();
                 // Refill this stage with the tile NS ahead.
                 if (ld.h < hend) {
@@ -456,17 +513,17 @@ __global__ void __launch_bounds__(MKFor<G>::NW * 32, 1)
                 }
             } else if (h == hfirst) {
                 const int64_t rec = (int64_t)c * NW + warp;  // this slab continues in an earlier warp
-                store_mma_state<G>(S, l2, a.warp_o + rec * G * kHeadDim, a.warp_ml + rec * G * 2, lane);
+                store_mma_state<NT>(S, l2, a.warp_o + rec * NC * kHeadDim, a.warp_ml + rec * NC * 2, NC, lane);
                 if (lane == 0) {
                     seg_first[warp] = h;
                     seg_p0[2 * warp] = p0h;
                     seg_p1[2 * warp] = p1h;
                 }
             } else if (FUSED) {
-                write_mma_out<G>(a, S, l2, b, g, lane);  // the whole slab lies in this warp's range
+                write_mma_out<G, NT>(a, S, l2, b, g, NC, lane);  // the whole slab lies in this warp's range
             } else {
                 const int64_t slot = (int64_t)c + h;  // the whole slab lies in this warp's range
-                store_mma_state<G>(S, l2, a.work_o + slot * G * kHeadDim, a.work_ml + slot * G * 2, lane);
+                store_mma_state<NT>(S, l2, a.work_o + slot * NC * kHeadDim, a.work_ml + slot * NC * 2, NC, lane);
             }
         }
 
@@ -486,36 +543,44 @@ __global__ void __launch_bounds__(MKFor<G>::NW * 32, 1)
     // final state goes there. Then the CTA merges, all warps sharing the work.
     __syncwarp();
     if (have_last)
-        store_mma_state<G>(S, l2, reinterpret_cast<float*>(my_ring), reinterpret_cast<float*>(my_ring) + G * kHeadDim,
-                           lane);
+        store_mma_state<NT>(S, l2, reinterpret_cast<float*>(my_ring), reinterpret_cast<float*>(my_ring) + NC * kHeadDim,
+                            NC, lane);
     __syncthreads();
     pdl_wait();  // the merges write the workspace and out: the previous kernel must be done with them
-    cta_tail<G, NW, FUSED>(a, smem, C::kWarpRing, seg_first, c, R, warp, lane);
+    cta_tail<G, NW, FUSED, NCC>(a, smem, C::kWarpRing, seg_first, c, R, warp, lane);
 }
 
-template <int G, bool FUSED>
+template <int G, int NT, bool FUSED, bool MULTI>
 cudaError_t launch_mma_g(const DecodeArgs& a, const CacheMaps& maps, const DecodeConfig& cfg, cudaStream_t st)
 {
-    return launch_pdl(decode_mma_kernel<G, FUSED>, cfg.nctas, MKFor<G>::NW * 32, cfg.smem_bytes, st, a, maps);
+    return launch_pdl(decode_mma_kernel<G, NT, FUSED, MULTI>, cfg.nctas, MKFor<G, NT>::NW * 32, cfg.smem_bytes, st, a,
+                      maps);
 }
 
-template <int G>
+// Launch configuration of the tensor-core kernel with NT column tiles (the
+// multi-query kernel, NT = 2, exists fused only).
+template <int G, int NT>
 cudaError_t config_mma_g(int B, DecodeConfig* cfg)
 {
-    using C = MKFor<G>;
+    using C = MKFor<G, NT>;
     const int smem = C::bytes(B);
     cudaError_t e;
-    if ((e = cudaFuncSetAttribute(decode_mma_kernel<G, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) !=
-        cudaSuccess)
-        return e;
-    if ((e = cudaFuncSetAttribute(decode_mma_kernel<G, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) !=
-        cudaSuccess)
+    if constexpr (NT == 1) {
+        if ((e = cudaFuncSetAttribute(decode_mma_kernel<G, NT, false, false>,
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess)
+            return e;
+        if ((e = cudaFuncSetAttribute(decode_mma_kernel<G, NT, true, false>,
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess)
+            return e;
+    }
+    if ((e = cudaFuncSetAttribute(decode_mma_kernel<G, NT, true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  smem)) != cudaSuccess)
         return e;
     int dev = 0, sms = 0, per_sm = 0;
     if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
     if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-    if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_mma_kernel<G, true>, C::NW * 32, smem)) !=
-        cudaSuccess)
+    if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_mma_kernel<G, NT, true, true>, C::NW * 32,
+                                                           smem)) != cudaSuccess)
         return e;
     if (per_sm < 1) return cudaErrorInvalidConfiguration;
     cfg->nctas = sms * per_sm;
@@ -560,36 +625,49 @@ cudaError_t make_cache_maps(const void* Kc, const void* Vc, int64_t rows, CacheM
     return cudaSuccess;
 }
 
-cudaError_t decode_config_mma(int G, int B, DecodeConfig* cfg)
+cudaError_t decode_config_mma(int G, int B, int NT, DecodeConfig* cfg)
 {
-    if (B < 1 || B > kMaxB) return cudaErrorInvalidValue;
+    if (B < 1 || B > kMaxB || NT < 1 || NT > 2) return cudaErrorInvalidValue;
+#define DKV_CFG_CASE(g) \
+    case g: return NT == 1 ? config_mma_g<g, 1>(B, cfg) : config_mma_g<g, 2>(B, cfg);
     switch (G) {
-        case 1: return config_mma_g<1>(B, cfg);
-        case 2: return config_mma_g<2>(B, cfg);
-        case 3: return config_mma_g<3>(B, cfg);
-        case 4: return config_mma_g<4>(B, cfg);
-        case 5: return config_mma_g<5>(B, cfg);
-        case 6: return config_mma_g<6>(B, cfg);
-        case 7: return config_mma_g<7>(B, cfg);
-        case 8: return config_mma_g<8>(B, cfg);
+        DKV_CFG_CASE(1)
+        DKV_CFG_CASE(2)
+        DKV_CFG_CASE(3)
+        DKV_CFG_CASE(4)
+        DKV_CFG_CASE(5)
+        DKV_CFG_CASE(6)
+        DKV_CFG_CASE(7)
+        DKV_CFG_CASE(8)
         default: return cudaErrorInvalidValue;
     }
+#undef DKV_CFG_CASE
 }
 
 template <bool FUSED>
 static cudaError_t launch_mma_any(const DecodeArgs& a, const CacheMaps& maps, const DecodeConfig& cfg, cudaStream_t st)
 {
+    // The decode step (Q = 1) takes the kernels with the G columns fixed at
+    // compile time; multi-query calls the fused ones with one or two column tiles.
+    const bool multi = a.Q > 1, two = a.NC > 8;
+    if (multi && !FUSED) return cudaErrorInvalidValue;
+#define DKV_LAUNCH_CASE(g)                                                                        \
+    case g:                                                                                       \
+        return !multi ? launch_mma_g<g, 1, FUSED, false>(a, maps, cfg, st)                        \
+                      : (two ? launch_mma_g<g, 2, true, true>(a, maps, cfg, st)                   \
+                             : launch_mma_g<g, 1, true, true>(a, maps, cfg, st));
     switch (a.G) {
-        case 1: return launch_mma_g<1, FUSED>(a, maps, cfg, st);
-        case 2: return launch_mma_g<2, FUSED>(a, maps, cfg, st);
-        case 3: return launch_mma_g<3, FUSED>(a, maps, cfg, st);
-        case 4: return launch_mma_g<4, FUSED>(a, maps, cfg, st);
-        case 5: return launch_mma_g<5, FUSED>(a, maps, cfg, st);
-        case 6: return launch_mma_g<6, FUSED>(a, maps, cfg, st);
-        case 7: return launch_mma_g<7, FUSED>(a, maps, cfg, st);
-        case 8: return launch_mma_g<8, FUSED>(a, maps, cfg, st);
+        DKV_LAUNCH_CASE(1)
+        DKV_LAUNCH_CASE(2)
+        DKV_LAUNCH_CASE(3)
+        DKV_LAUNCH_CASE(4)
+        DKV_LAUNCH_CASE(5)
+        DKV_LAUNCH_CASE(6)
+        DKV_LAUNCH_CASE(7)
+        DKV_LAUNCH_CASE(8)
         default: return cudaErrorInvalidValue;
     }
+#undef DKV_LAUNCH_CASE
 }
 
 cudaError_t launch_decode_mma_partial(const DecodeArgs& a, const CacheMaps& maps, const DecodeConfig& cfg,

@@ -70,7 +70,13 @@ struct DecodeArgs {
     int append;             // 1 when k_new/v_new are given
     float qscale;           // softmax scale * log2(e)
     int nctas;              // CTAs of the split-K grid: the row partition's part count
+    int Q;                  // queries per sequence (1 for the decode step); q and out are [B][Q][H][128]
+    int NC;                 // columns per slab: Q * G; partial records hold NC rows of 128 + 2 floats
 };
+
+// Most columns (queries x group heads) one decode call handles; the plan's
+// split-K workspace and arrival counters are sized for this many.
+constexpr int kMaxCols = 16;
 
 struct DecodeConfig {
     int nctas;        // grid of the partial kernel
@@ -84,6 +90,12 @@ struct DecodeConfig {
 inline int64_t decode_workspace_floats(const DecodeConfig& c, int G, int heads_per_layer) {
     const int64_t records = (int64_t)c.nctas + heads_per_layer + (int64_t)c.nctas * c.nwarps;
     return records * G * (128 + 2);
+}
+// The same for a workspace shared by kernels of up to `nctas` CTAs of up to
+// `nwarps` warps handling up to `cols` columns.
+inline int64_t decode_workspace_floats(int nctas, int nwarps, int cols, int heads_per_layer) {
+    const int64_t records = (int64_t)nctas + heads_per_layer + (int64_t)nctas * nwarps;
+    return records * cols * (128 + 2);
 }
 // Grid and shared memory of the partial kernel for group size G on this device.
 cudaError_t decode_config(int G, int B, DecodeConfig* cfg);
@@ -103,7 +115,9 @@ struct CacheMaps {
 };
 constexpr int64_t kMaxMmaRows = ((int64_t)1 << 31) - 16;
 cudaError_t make_cache_maps(const void* Kc, const void* Vc, int64_t rows, CacheMaps* maps);
-cudaError_t decode_config_mma(int G, int B, DecodeConfig* cfg);
+// Launch configuration of the tensor-core kernel with NT tiles of 8 columns:
+// NT = 1 for up to 8 columns (the decode step), 2 for up to 16 (multi-query).
+cudaError_t decode_config_mma(int G, int B, int NT, DecodeConfig* cfg);
 cudaError_t launch_decode_mma_partial(const DecodeArgs& a, const CacheMaps& maps, const DecodeConfig& cfg,
                                       cudaStream_t st);
 cudaError_t launch_decode_mma_fused(const DecodeArgs& a, const CacheMaps& maps, const DecodeConfig& cfg,

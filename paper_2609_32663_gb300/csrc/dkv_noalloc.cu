@@ -134,6 +134,8 @@ extern "C" dkv_status dkv_decode_attn_noalloc(const dkv_shape* s, int32_t B, int
     a.H = s->H;
     a.Hkv = s->H_kv;
     a.G = G;
+    a.Q = 1;
+    a.NC = G;
     a.reserve = reserve_rows;
     a.append = k_new ? 1 : 0;
     const float sc = scale > 0.f ? scale : 1.0f / std::sqrt((float)dkv::kHeadDim);

@@ -26,7 +26,7 @@ DKV_DEV_TMA_TIMEOUT = 0x2
 EXPORTS = ("dkv_last_error", "dkv_map_pattern", "dkv_plan_dense", "dkv_plan_query", "dkv_plan_read",
            "dkv_compact", "dkv_decode_attn", "dkv_decode_partial", "dkv_decode_combine", "dkv_advance",
            "dkv_plan_status", "dkv_free", "dkv_decode_attn_noalloc", "dkv_budget", "dkv_topk_workspace_bytes",
-           "dkv_topk_mask")
+           "dkv_topk_mask", "dkv_decode_multi")
 
 
 class DkvError(RuntimeError):
@@ -90,6 +90,8 @@ def lib(path: str | None = None):
     L.dkv_compact.argtypes = [V, V, V, I64, V, V, V]
     L.dkv_decode_attn.restype = ctypes.c_int
     L.dkv_decode_attn.argtypes = [V, I32, V, V, V, V, V, V, ctypes.c_float, V, V]
+    L.dkv_decode_multi.restype = ctypes.c_int
+    L.dkv_decode_multi.argtypes = [V, I32, V, I32, V, V, V, ctypes.c_float, V, V]
     L.dkv_decode_partial.restype = ctypes.c_int
     L.dkv_decode_partial.argtypes = [V, I32, V, V, V, V, V, V, ctypes.c_float, V]
     L.dkv_decode_combine.restype = ctypes.c_int
@@ -213,6 +215,14 @@ def dkv_decode_attn(plan: Plan, layer: int, q, k_new, v_new, n_appended, Kc, Vc,
     _check(lib().dkv_decode_attn(plan, int(layer), _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(n_appended),
                                  _ptr(Kc), _ptr(Vc), ctypes.c_float(scale), _ptr(out), _stream(stream)),
            "dkv_decode_attn")
+
+
+def dkv_decode_multi(plan: Plan, layer: int, q, num_queries: int, n_appended, Kc, Vc, out, scale: float = 0.0,
+                     stream=None):
+    """num_queries queries per sequence over the same compressed rows: q bf16
+    [B][Q][H][128] -> out fp32 [B][Q][H][128]."""
+    _check(lib().dkv_decode_multi(plan, int(layer), _ptr(q), int(num_queries), _ptr(n_appended), _ptr(Kc), _ptr(Vc),
+                                  ctypes.c_float(scale), _ptr(out), _stream(stream)), "dkv_decode_multi")
 
 
 def dkv_decode_partial(plan: Plan, layer: int, q, k_new, v_new, n_appended, Kc, Vc, scale: float = 0.0,
