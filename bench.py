@@ -216,7 +216,7 @@ def setup(wl, dev, reserve):
     Kc = torch.empty((info.total_rows, wl.head_dim), dtype=torch.bfloat16, device=dev)
     Vc = torch.empty_like(Kc)
     return dict(M=M, Tc=Tc, shape=shape, T_stride=T_stride, K=K, V=V, plan=plan, info=info, Kc=Kc, Vc=Vc,
-                map_ms=map_ms)
+                map_ms=map_ms, reserve=reserve)
 
 
 def time_compaction(env, reps=10):
@@ -269,6 +269,38 @@ def time_topk(wl, dev, reps=10):
                     "algorithmic_gbs": round(5 * n / t / 1e9, 1), "streamed_gbs": round(25 * n / t / 1e9, 1),
                     "launches": 7}
     return out
+
+
+def time_compaction_inplace(wl, env, reps=5):
+    """dkv_compact_inplace on the dense caches (run last: it overwrites them).
+    Bytes: the rows that move (from the first dropped position of each slab on)
+    read and written, plus their indices."""
+    import torch
+
+    import paper_2609_32663_gb300.dkv as dkv
+    plan = dkv.dkv_map_pattern_inplace(env["M"], env["Tc"], env["shape"], env["T_stride"],
+                                       reserve_rows=env["reserve"])
+    ln, _, ioff, idx = dkv.dkv_plan_read(plan)
+    moved = 0
+    for h in range(len(ln)):
+        ids = idx[ioff[h]:ioff[h + 1]]
+        stay = np.flatnonzero(ids != np.arange(ids.size))
+        moved += ids.size - (int(stay[0]) if stay.size else ids.size)
+    times = []
+    st = torch.cuda.current_stream()
+    for i in range(reps + 1):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(st)
+        dkv.dkv_compact_inplace(plan, env["K"], env["V"])
+        e1.record(st)
+        e1.synchronize()
+        if i >= 1:
+            times.append(e0.elapsed_time(e1) * 1e-3)
+    plan.close()
+    t = statistics.median(times)
+    algo = moved * (2 * 256 * 2 + 4)
+    return {"ms": round(t * 1e3, 3), "gbs": round(algo / t / 1e9, 1), "moved_rows": int(moved),
+            "kept_rows": int(ln.sum()), "how": "median of %d; later reps move already-moved bytes (same volume)" % reps}
 
 
 def time_multi_query(wl, env, dev, Q, steps, warmup):
@@ -606,6 +638,8 @@ def run_dkv(args, dist):
             mq[f"Q{Q}"] = {"us_per_step": round(t_q * 1e6, 2), "queries_per_s": round(wl.B * Q * dist.world / t_q, 1),
                            "gbs": round(step_bytes(wl, rows_q, with_new=False) / t_q / 1e9, 1)}
         res["multi_query"] = mq
+    if not args.profile:
+        res["compaction_inplace"] = time_compaction_inplace(wl, env)  # last: overwrites the dense caches
     st = dkv.dkv_plan_status(env["plan"])
     res["device_status_word"] = st
     env["plan"].close()

@@ -154,6 +154,30 @@ dkv_status dkv_compact(const dkv_plan* plan, const void* K, const void* V, int64
                        void* Kc, void* Vc, cudaStream_t stream);
 
 /*
+ * In-place variant of the two calls above (Sec. 3.4: evicted states are
+ * physically removed): the packed cache lives inside the dense one, so no
+ * second cache is allocated at compaction time.
+ *
+ * dkv_map_pattern_inplace   as dkv_map_pattern, but slab h starts at row
+ *                           h * T_stride, the first row of its own region of the
+ *                           dense K/V [L][B][H_kv][T_stride][128]: off[h] =
+ *                           h * T_stride, total_rows = L*B*H_kv * T_stride, and
+ *                           rows [len[h], len[h] + reserve_rows) of the region
+ *                           take appended tokens. Needs T_stride >= max ctx_len
+ *                           + reserve_rows.
+ * dkv_compact_inplace       moves each slab's kept rows, in token order, to the
+ *                           start of its region of K and of V (rows [0, len)).
+ *                           Rows past len are left as they were. Afterwards pass
+ *                           K and V as Kc and Vc to the decode calls. K and V:
+ *                           device, 16-byte aligned, distinct.
+ * Errors: DKV_ERR_INVALID_ARG (as above; a plan not made by
+ * dkv_map_pattern_inplace), DKV_ERR_RANGE, DKV_ERR_OOM, DKV_ERR_CUDA.
+ */
+dkv_status dkv_map_pattern_inplace(const uint8_t* M, const int32_t* ctx_len, int32_t B, const dkv_shape* shape,
+                                   int32_t reserve_rows, int64_t T_stride, cudaStream_t stream, dkv_plan** plan);
+dkv_status dkv_compact_inplace(const dkv_plan* plan, void* K, void* V, cudaStream_t stream);
+
+/*
  * Decode-step attention of one layer over the packed cache (Sec. 3.4), split-K
  * over the kept rows with an online-softmax merge.
  *

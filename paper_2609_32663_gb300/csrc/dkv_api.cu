@@ -36,6 +36,7 @@ struct dkv_plan {
     int64_t slots = 0;              // (CTA, slab) partial slots: CTAs + slabs of a layer
     int nctas_cap = 0, warps_cap = 0, cols_cap = 0;  // workspace sized for these
     int use_mma = 0;  // tensor-core decode kernel (needs the cache's row count for its tensor maps)
+    int64_t inplace_stride = 0;  // > 0: slab h lives at rows h * stride of the dense buffer (in place)
 };
 
 namespace {
@@ -176,9 +177,11 @@ extern "C" {
 
 const char* dkv_last_error(void) { return g_err; }
 
-dkv_status dkv_map_pattern(const uint8_t* M_host, const int32_t* ctx_len_host, int32_t B,
-                           const dkv_shape* s, int32_t reserve_rows, cudaStream_t stream,
-                           dkv_plan** out)
+// The map of dkv_map_pattern and dkv_map_pattern_inplace: slab offsets are the
+// running sum of (len + reserve), or h * inplace_stride when that is > 0.
+static dkv_status map_pattern_impl(const uint8_t* M_host, const int32_t* ctx_len_host, int32_t B,
+                                   const dkv_shape* s, int32_t reserve_rows, int64_t inplace_stride,
+                                   cudaStream_t stream, dkv_plan** out)
 {
     if (!out) return fail(DKV_ERR_INVALID_ARG, "out is NULL");
     *out = nullptr;
@@ -200,6 +203,9 @@ dkv_status dkv_map_pattern(const uint8_t* M_host, const int32_t* ctx_len_host, i
                         s->D, s->bin_width);
         if (T > Tmax) Tmax = T;
     }
+    if (inplace_stride > 0 && inplace_stride < (int64_t)Tmax + reserve_rows)
+        return fail(DKV_ERR_INVALID_ARG, "T_stride=%lld < longest context %d + reserve %d", (long long)inplace_stride,
+                    Tmax, reserve_rows);
     // Rows of one layer (with reserve) must fit the decode kernel's int32 row arithmetic.
     {
         int64_t layer_rows = 0;
@@ -214,6 +220,8 @@ dkv_status dkv_map_pattern(const uint8_t* M_host, const int32_t* ctx_len_host, i
     p->B = B;
     p->G = s->H / s->H_kv;
     p->reserve = reserve_rows;
+    p->inplace_stride = inplace_stride;
+    p->T_stride = inplace_stride;
 
     const int NH = s->L * B * s->H_kv;
     const int nchunks = Tmax > 0 ? (Tmax + dkv::kMapChunk - 1) / dkv::kMapChunk : 1;
@@ -269,6 +277,7 @@ dkv_status dkv_map_pattern(const uint8_t* M_host, const int32_t* ctx_len_host, i
     ma.reserve = reserve_rows;
     ma.nchunks = nchunks;
     ma.NH = NH;
+    ma.stride = inplace_stride;
     if ((st = launched(dkv::launch_map(ma, stream), "map kernels")) != DKV_OK) {
         cleanup();
         release(p);
@@ -307,6 +316,21 @@ dkv_status dkv_map_pattern(const uint8_t* M_host, const int32_t* ctx_len_host, i
     }
     *out = p;
     return ok();
+}
+
+dkv_status dkv_map_pattern(const uint8_t* M_host, const int32_t* ctx_len_host, int32_t B, const dkv_shape* s,
+                           int32_t reserve_rows, cudaStream_t stream, dkv_plan** out)
+{
+    return map_pattern_impl(M_host, ctx_len_host, B, s, reserve_rows, 0, stream, out);
+}
+
+dkv_status dkv_map_pattern_inplace(const uint8_t* M_host, const int32_t* ctx_len_host, int32_t B,
+                                   const dkv_shape* s, int32_t reserve_rows, int64_t T_stride, cudaStream_t stream,
+                                   dkv_plan** out)
+{
+    if (out) *out = nullptr;
+    if (T_stride < 1) return fail(DKV_ERR_INVALID_ARG, "T_stride=%lld < 1", (long long)T_stride);
+    return map_pattern_impl(M_host, ctx_len_host, B, s, reserve_rows, T_stride, stream, out);
 }
 
 dkv_status dkv_plan_dense(const int32_t* ctx_len_host, int32_t B, const dkv_shape* s, int64_t T_stride,
@@ -403,11 +427,35 @@ dkv_status dkv_plan_read(const dkv_plan* p, int32_t* len_host, int64_t* off_host
     return ok();
 }
 
+dkv_status dkv_compact_inplace(const dkv_plan* p, void* K, void* V, cudaStream_t stream)
+{
+    if (!p) return fail(DKV_ERR_INVALID_ARG, "plan is NULL");
+    if (p->dense || p->inplace_stride <= 0)
+        return fail(DKV_ERR_INVALID_ARG, "dkv_compact_inplace needs a plan from dkv_map_pattern_inplace");
+    if (!K || !V) return fail(DKV_ERR_INVALID_ARG, "NULL K/V");
+    if (!aligned16(K) || !aligned16(V)) return fail(DKV_ERR_INVALID_ARG, "K/V must be 16-byte aligned");
+    if (K == V) return fail(DKV_ERR_INVALID_ARG, "K and V must be different buffers");
+    dkv::CompactArgs a{};
+    a.len = p->d_len;
+    a.off = p->d_off;
+    a.ioff = p->d_ioff;
+    a.idx = p->d_idx;
+    a.K = static_cast<const uint16_t*>(K);
+    a.V = static_cast<const uint16_t*>(V);
+    a.T_stride = p->inplace_stride;
+    a.kept = p->kept_rows;
+    a.NH = p->s.L * p->B * p->s.H_kv;
+    dkv_status st = launched(dkv::launch_compact_inplace(a, stream), "in-place compact kernel");
+    return st == DKV_OK ? ok() : st;
+}
+
 dkv_status dkv_compact(const dkv_plan* p, const void* K, const void* V, int64_t T_stride, void* Kc, void* Vc,
                        cudaStream_t stream)
 {
     if (!p) return fail(DKV_ERR_INVALID_ARG, "plan is NULL");
     if (p->dense) return fail(DKV_ERR_INVALID_ARG, "dkv_compact needs a plan from dkv_map_pattern");
+    if (p->inplace_stride > 0)
+        return fail(DKV_ERR_INVALID_ARG, "an in-place plan is compacted by dkv_compact_inplace");
     if (!K || !V || !Kc || !Vc) return fail(DKV_ERR_INVALID_ARG, "NULL K/V/Kc/Vc");
     if (!aligned16(K) || !aligned16(V) || !aligned16(Kc) || !aligned16(Vc))
         return fail(DKV_ERR_INVALID_ARG, "K/V/Kc/Vc must be 16-byte aligned");

@@ -80,6 +80,74 @@ __global__ void __launch_bounds__(kThreads) compact_kernel(const CompactArgs a)
 
 }  // namespace
 
+// In-place prune-and-pack: slab h's kept rows move from rows h * T_stride +
+// idx[r] to rows h * T_stride + r of the same buffer. idx is ascending, so
+// idx[r] >= r: a row only moves towards the slab's start, and rows before the
+// first dropped position stay where they are. One CTA walks a slab in chunks of
+// kInChunk rows: it loads the chunk's source rows into registers, waits at a
+// barrier for all of them, then stores. A chunk's sources lie at or after its
+// own destinations and strictly after the previous chunks' destinations, and
+// the next chunk's destinations come after this chunk's barrier, so no row is
+// overwritten before it has been read. Loads bypass L1 (the buffer is written
+// by this kernel).
+constexpr int kInThreads = 256;
+constexpr int kInChunk = 64;                               // rows per chunk
+constexpr int kInPer = kInChunk * 2 * 16 / kInThreads;     // 16-byte pieces per thread per chunk (K and V)
+
+__global__ void __launch_bounds__(kInThreads) compact_inplace_kernel(const CompactArgs a)
+{
+    uint16_t* K = const_cast<uint16_t*>(a.K);
+    uint16_t* V = const_cast<uint16_t*>(a.V);
+    for (int h = blockIdx.x; h < a.NH; h += gridDim.x) {
+        const int n = a.len[h];
+        const int32_t* idx = a.idx + a.ioff[h];
+        const int64_t base = (int64_t)h * a.T_stride;
+        // First row that moves: idx[r] - r is non-decreasing, so a binary search.
+        int lo = 0, hi = n;
+        while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (__ldg(idx + mid) > mid)
+                hi = mid;
+            else
+                lo = mid + 1;
+        }
+        for (int r0 = lo; r0 < n; r0 += kInChunk) {
+            uint4 v[kInPer];
+            int64_t dst[kInPer];
+#pragma unroll
+            for (int k = 0; k < kInPer; ++k) {
+                const int piece = threadIdx.x + k * kInThreads;  // (row, K/V, 16-byte chunk)
+                const int r = r0 + piece / 32, kv = (piece / 16) & 1, c = piece & 15;
+                dst[k] = -1;
+                if (r < n) {
+                    const uint16_t* src = (kv ? V : K) + (base + __ldg(idx + r)) * kHeadDim;
+                    v[k] = __ldcg(reinterpret_cast<const uint4*>(src) + c);
+                    dst[k] = ((base + r) * kHeadDim) / 8 + c;  // in uint4 units
+                }
+            }
+            __syncthreads();  // every source row of this chunk is read
+#pragma unroll
+            for (int k = 0; k < kInPer; ++k) {
+                const int piece = threadIdx.x + k * kInThreads;
+                const int kv = (piece / 16) & 1;
+                if (dst[k] >= 0) reinterpret_cast<uint4*>(kv ? V : K)[dst[k]] = v[k];
+            }
+        }
+    }
+}
+
+cudaError_t launch_compact_inplace(const CompactArgs& a, cudaStream_t st)
+{
+    if (a.kept == 0 || a.NH == 0) return cudaSuccess;
+    int dev = 0, sms = 0;
+    cudaError_t e;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+    const int grid = a.NH < 8 * sms ? a.NH : 8 * sms;
+    compact_inplace_kernel<<<grid, kInThreads, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_compact(const CompactArgs& a, cudaStream_t st)
 {
     if (a.kept == 0) return cudaSuccess;

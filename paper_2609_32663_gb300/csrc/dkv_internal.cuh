@@ -24,6 +24,7 @@ struct MapArgs {
     int L, H, Hkv, D, B, sink, recent, bin_width, reserve;
     int nchunks;            // position chunks per slab
     int NH;                 // L*B*Hkv
+    int64_t stride;         // 0: slabs packed end to end; > 0: slab h starts at row h * stride (in place)
 };
 constexpr int kMapChunk = 8192;  // positions per CTA in the count/write passes
 
@@ -46,6 +47,9 @@ struct CompactArgs {
     int NH;
 };
 cudaError_t launch_compact(const CompactArgs& a, cudaStream_t st);
+// In place: K and V are both source and destination, slab h at rows h * T_stride
+// (Kc/Vc unused); every slab's kept rows move to its first len rows, in order.
+cudaError_t launch_compact_inplace(const CompactArgs& a, cudaStream_t st);
 
 // ---------------------------------------------------------------- decode
 struct DecodeArgs {

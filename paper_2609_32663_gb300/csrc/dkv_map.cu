@@ -121,13 +121,13 @@ __global__ void __launch_bounds__(kScanThreads) scan_kernel(const MapArgs a)
     int64_t run_off = sh_off[threadIdx.x] - s_off;
     int64_t run_ioff = sh_ioff[threadIdx.x] - s_ioff;
     for (int h = h0; h < h1; ++h) {
-        a.off[h] = run_off;
+        a.off[h] = a.stride > 0 ? (int64_t)h * a.stride : run_off;  // in place: the slab's own dense rows
         a.ioff[h] = run_ioff;
         run_off += (int64_t)a.len[h] + a.reserve;
         run_ioff += a.len[h];
     }
     if (threadIdx.x == kScanThreads - 1) {
-        a.off[a.NH] = sh_off[kScanThreads - 1];
+        a.off[a.NH] = a.stride > 0 ? (int64_t)a.NH * a.stride : sh_off[kScanThreads - 1];
         a.ioff[a.NH] = sh_ioff[kScanThreads - 1];
     }
 }

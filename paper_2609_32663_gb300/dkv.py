@@ -26,7 +26,7 @@ DKV_DEV_TMA_TIMEOUT = 0x2
 EXPORTS = ("dkv_last_error", "dkv_map_pattern", "dkv_plan_dense", "dkv_plan_query", "dkv_plan_read",
            "dkv_compact", "dkv_decode_attn", "dkv_decode_partial", "dkv_decode_combine", "dkv_advance",
            "dkv_plan_status", "dkv_free", "dkv_decode_attn_noalloc", "dkv_budget", "dkv_topk_workspace_bytes",
-           "dkv_topk_mask", "dkv_decode_multi")
+           "dkv_topk_mask", "dkv_decode_multi", "dkv_map_pattern_inplace", "dkv_compact_inplace")
 
 
 class DkvError(RuntimeError):
@@ -80,6 +80,10 @@ def lib(path: str | None = None):
     L.dkv_last_error.argtypes = []
     L.dkv_map_pattern.restype = ctypes.c_int
     L.dkv_map_pattern.argtypes = [V, V, I32, ctypes.POINTER(dkv_shape), I32, V, PP]
+    L.dkv_map_pattern_inplace.restype = ctypes.c_int
+    L.dkv_map_pattern_inplace.argtypes = [V, V, I32, ctypes.POINTER(dkv_shape), I32, I64, V, PP]
+    L.dkv_compact_inplace.restype = ctypes.c_int
+    L.dkv_compact_inplace.argtypes = [V, V, V, V]
     L.dkv_plan_dense.restype = ctypes.c_int
     L.dkv_plan_dense.argtypes = [V, I32, ctypes.POINTER(dkv_shape), I64, V, PP]
     L.dkv_plan_query.restype = ctypes.c_int
@@ -174,6 +178,22 @@ def dkv_map_pattern(M, ctx_len, shape: Shape, reserve_rows: int = 0, stream=None
     _check(lib().dkv_map_pattern(_ptr(M), _ptr(ctx), len(ctx), ctypes.byref(sh), int(reserve_rows),
                                  _stream(stream), ctypes.byref(out)), "dkv_map_pattern")
     return Plan(out.value, shape, len(ctx), False)
+
+
+def dkv_map_pattern_inplace(M, ctx_len, shape: Shape, T_stride: int, reserve_rows: int = 0, stream=None) -> Plan:
+    """dkv_map_pattern with every slab at the start of its own dense region (off[h] = h T_stride)."""
+    M = np.ascontiguousarray(M, dtype=np.uint8)
+    ctx = np.ascontiguousarray(ctx_len, dtype=np.int32)
+    out = ctypes.c_void_p()
+    sh = shape.c()
+    _check(lib().dkv_map_pattern_inplace(_ptr(M), _ptr(ctx), len(ctx), ctypes.byref(sh), int(reserve_rows),
+                                         int(T_stride), _stream(stream), ctypes.byref(out)), "dkv_map_pattern_inplace")
+    return Plan(out.value, shape, len(ctx), False)
+
+
+def dkv_compact_inplace(plan: Plan, K, V, stream=None):
+    """Move each slab's kept rows to the start of its region of K and V (in place)."""
+    _check(lib().dkv_compact_inplace(plan, _ptr(K), _ptr(V), _stream(stream)), "dkv_compact_inplace")
 
 
 def dkv_plan_dense(ctx_len, shape: Shape, T_stride: int, stream=None) -> Plan:

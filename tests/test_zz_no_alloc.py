@@ -95,11 +95,14 @@ def test_noalloc_allocates_nothing(case):
     torch.cuda.synchronize()
     free0 = torch.cuda.mem_get_info()[0]
     torch_bytes = torch.cuda.memory_allocated()
-    for layer in range(wl.L):
-        dkv.dkv_decode_attn_noalloc(c.sh, wl.B, layer, c.reserve, d_len, d_off, d_ioff, q, None, None, None,
+    calls = 64
+    for i in range(calls):
+        dkv.dkv_decode_attn_noalloc(c.sh, wl.B, i % wl.L, c.reserve, d_len, d_off, d_ioff, q, None, None, None,
                                     c.Kc, c.Vc, out)
     torch.cuda.synchronize()
-    assert torch.cuda.mem_get_info()[0] == free0
+    # Device-wide free memory also moves with the driver's own bookkeeping, so the
+    # check is for growth: an allocation per call would lose >= 64 x its size.
+    assert free0 - torch.cuda.mem_get_info()[0] < (2 << 20)
     assert torch.cuda.memory_allocated() == torch_bytes
 
 
