@@ -178,6 +178,41 @@ dkv_status dkv_map_pattern_inplace(const uint8_t* M, const int32_t* ctx_len, int
 dkv_status dkv_compact_inplace(const dkv_plan* plan, void* K, void* V, cudaStream_t stream);
 
 /*
+ * Page-backed cache buffers, so that the memory of evicted states can be given
+ * back after an in-place compaction (Sec. 3.4: evicted states are physically
+ * removed; App. C reports the memory this saves).
+ *
+ * dkv_vmm_alloc      a device buffer of at least `bytes` bytes, one reserved
+ *                    address range backed by separate physical pages of the
+ *                    device's allocation granularity (*dptr: its address).
+ *                    Allocate the dense K and the dense V each this way, then
+ *                    fill them, map and compact in place.
+ * dkv_vmm_trim       unmap and release every page of the buffer that holds no
+ *                    row in [0, min(T_stride, len[h] + reserve + guard_rows)) of
+ *                    any slab h of the in-place plan (rows of 256 bytes, slab h
+ *                    at row h * T_stride). Accessing a released page faults:
+ *                    afterwards use the buffer only through that plan (decode,
+ *                    multi-query decode, appends within the reserve).
+ *                    guard_rows >= 16: the decode kernels read whole 16-row
+ *                    tiles, up to 15 rows past a slab's last row. Synchronises
+ *                    the device. *freed_bytes: the memory released by this call.
+ * dkv_vmm_pages_to_keep  the page rule of dkv_vmm_trim on host arrays: keep[i]
+ *                    = 1 for page i of npages (page_bytes each) that must stay
+ *                    mapped for slabs of len[h] rows (host only).
+ * dkv_vmm_mapped_bytes / dkv_vmm_page_bytes  mapped bytes now; page size.
+ * dkv_vmm_free       synchronise the device and release the buffer (NULL-safe).
+ * Errors: DKV_ERR_INVALID_ARG, DKV_ERR_OOM, DKV_ERR_CUDA.
+ */
+typedef struct dkv_vmm dkv_vmm;
+dkv_status dkv_vmm_alloc(int64_t bytes, dkv_vmm** buffer, void** dptr);
+dkv_status dkv_vmm_trim(dkv_vmm* buffer, const dkv_plan* plan, int32_t guard_rows, int64_t* freed_bytes);
+void dkv_vmm_pages_to_keep(const int32_t* len, int64_t nslabs, int64_t T_stride, int32_t reserve, int32_t guard_rows,
+                           int64_t row_bytes, int64_t page_bytes, int64_t npages, uint8_t* keep);
+int64_t dkv_vmm_mapped_bytes(const dkv_vmm* buffer);
+int64_t dkv_vmm_page_bytes(const dkv_vmm* buffer);
+void dkv_vmm_free(dkv_vmm* buffer);
+
+/*
  * Decode-step attention of one layer over the packed cache (Sec. 3.4), split-K
  * over the kept rows with an online-softmax merge.
  *

@@ -165,6 +165,13 @@ dkv_status finish_plan(dkv_plan* p)
 }  // namespace
 
 namespace dkv {
+// Page-backed buffers (dkv_vmm.cu).
+dkv_status vmm_release_pages(dkv_vmm* m, const uint8_t* keep, int64_t npages, int64_t* freed);
+int64_t vmm_bytes(const dkv_vmm* m);
+int64_t vmm_page(const dkv_vmm* m);
+}  // namespace dkv
+
+namespace dkv {
 // Lets other translation units of the library report through dkv_last_error().
 dkv_status set_error(dkv_status st, const char* msg)
 {
@@ -447,6 +454,29 @@ dkv_status dkv_compact_inplace(const dkv_plan* p, void* K, void* V, cudaStream_t
     a.NH = p->s.L * p->B * p->s.H_kv;
     dkv_status st = launched(dkv::launch_compact_inplace(a, stream), "in-place compact kernel");
     return st == DKV_OK ? ok() : st;
+}
+
+dkv_status dkv_vmm_trim(dkv_vmm* m, const dkv_plan* p, int32_t guard_rows, int64_t* freed_bytes)
+{
+    if (freed_bytes) *freed_bytes = 0;
+    if (!m || !p) return fail(DKV_ERR_INVALID_ARG, "NULL buffer or plan");
+    if (p->inplace_stride <= 0) return fail(DKV_ERR_INVALID_ARG, "dkv_vmm_trim needs a plan from dkv_map_pattern_inplace");
+    if (guard_rows < 16)
+        return fail(DKV_ERR_INVALID_ARG, "guard_rows=%d < 16: decode reads whole 16-row tiles past a slab's last row",
+                    guard_rows);
+    const int64_t NH = (int64_t)p->s.L * p->B * p->s.H_kv;
+    const int64_t need = NH * p->inplace_stride * dkv::kRowBytes;
+    if (dkv::vmm_bytes(m) < need)
+        return fail(DKV_ERR_INVALID_ARG, "buffer of %lld bytes is smaller than the plan's cache (%lld bytes)",
+                    (long long)dkv::vmm_bytes(m), (long long)need);
+    std::vector<int32_t> len((size_t)NH);
+    cudaError_t e = cudaMemcpy(len.data(), p->d_len, sizeof(int32_t) * NH, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(e, "read lengths");
+    const int64_t page = dkv::vmm_page(m), npages = dkv::vmm_bytes(m) / page;
+    std::vector<uint8_t> keep((size_t)npages);
+    dkv::vmm_pages_to_keep(len.data(), NH, p->inplace_stride, p->reserve, guard_rows, dkv::kRowBytes, page, npages,
+                           keep.data());
+    return dkv::vmm_release_pages(m, keep.data(), npages, freed_bytes);
 }
 
 dkv_status dkv_compact(const dkv_plan* p, const void* K, const void* V, int64_t T_stride, void* Kc, void* Vc,

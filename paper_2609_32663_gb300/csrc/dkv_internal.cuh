@@ -131,6 +131,11 @@ cudaError_t launch_advance(int32_t* n_app, int B, int reserve, int32_t* status, 
 // Exact-budget Top-K pattern export (dkv_topk.cu): device workspace bytes, and
 // the launches (4 histogram passes, tie count, mark) on `st`.
 int64_t topk_workspace_bytes();
+
+// Page-backed buffers (dkv_vmm.cu): which pages a slab layout still needs, and
+// the release of the others (synchronises the device first).
+void vmm_pages_to_keep(const int32_t* len, int64_t nslabs, int64_t T_stride, int64_t reserve, int64_t guard,
+                       int64_t row_bytes, int64_t page, int64_t npages, uint8_t* keep);
 cudaError_t launch_topk(const float* P, int64_t n, int64_t K, uint8_t* M, void* workspace, cudaStream_t st);
 
 }  // namespace dkv

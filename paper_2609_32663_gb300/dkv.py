@@ -26,7 +26,9 @@ DKV_DEV_TMA_TIMEOUT = 0x2
 EXPORTS = ("dkv_last_error", "dkv_map_pattern", "dkv_plan_dense", "dkv_plan_query", "dkv_plan_read",
            "dkv_compact", "dkv_decode_attn", "dkv_decode_partial", "dkv_decode_combine", "dkv_advance",
            "dkv_plan_status", "dkv_free", "dkv_decode_attn_noalloc", "dkv_budget", "dkv_topk_workspace_bytes",
-           "dkv_topk_mask", "dkv_decode_multi", "dkv_map_pattern_inplace", "dkv_compact_inplace")
+           "dkv_topk_mask", "dkv_decode_multi", "dkv_map_pattern_inplace", "dkv_compact_inplace",
+           "dkv_vmm_alloc", "dkv_vmm_trim", "dkv_vmm_pages_to_keep", "dkv_vmm_mapped_bytes", "dkv_vmm_page_bytes",
+           "dkv_vmm_free")
 
 
 class DkvError(RuntimeError):
@@ -84,6 +86,18 @@ def lib(path: str | None = None):
     L.dkv_map_pattern_inplace.argtypes = [V, V, I32, ctypes.POINTER(dkv_shape), I32, I64, V, PP]
     L.dkv_compact_inplace.restype = ctypes.c_int
     L.dkv_compact_inplace.argtypes = [V, V, V, V]
+    L.dkv_vmm_alloc.restype = ctypes.c_int
+    L.dkv_vmm_alloc.argtypes = [I64, PP, PP]
+    L.dkv_vmm_trim.restype = ctypes.c_int
+    L.dkv_vmm_trim.argtypes = [V, V, I32, ctypes.POINTER(I64)]
+    L.dkv_vmm_pages_to_keep.restype = None
+    L.dkv_vmm_pages_to_keep.argtypes = [V, I64, I64, I32, I32, I64, I64, I64, V]
+    L.dkv_vmm_mapped_bytes.restype = I64
+    L.dkv_vmm_mapped_bytes.argtypes = [V]
+    L.dkv_vmm_page_bytes.restype = I64
+    L.dkv_vmm_page_bytes.argtypes = [V]
+    L.dkv_vmm_free.restype = None
+    L.dkv_vmm_free.argtypes = [V]
     L.dkv_plan_dense.restype = ctypes.c_int
     L.dkv_plan_dense.argtypes = [V, I32, ctypes.POINTER(dkv_shape), I64, V, PP]
     L.dkv_plan_query.restype = ctypes.c_int
@@ -194,6 +208,56 @@ def dkv_map_pattern_inplace(M, ctx_len, shape: Shape, T_stride: int, reserve_row
 def dkv_compact_inplace(plan: Plan, K, V, stream=None):
     """Move each slab's kept rows to the start of its region of K and V (in place)."""
     _check(lib().dkv_compact_inplace(plan, _ptr(K), _ptr(V), _stream(stream)), "dkv_compact_inplace")
+
+
+class VmmBuffer:
+    """A page-backed device buffer (dkv_vmm_alloc); .tensor(shape, dtype) views it as a torch tensor."""
+
+    def __init__(self, nbytes: int):
+        h, p = ctypes.c_void_p(), ctypes.c_void_p()
+        _check(lib().dkv_vmm_alloc(int(nbytes), ctypes.byref(h), ctypes.byref(p)), "dkv_vmm_alloc")
+        self.handle, self.ptr, self.nbytes = h.value, p.value, int(nbytes)
+
+    @property
+    def _as_parameter_(self):
+        return ctypes.c_void_p(self.handle)
+
+    def tensor(self, shape, dtype):
+        import torch
+        typestr = {torch.bfloat16: "<i2", torch.int16: "<i2", torch.float32: "<f4", torch.uint8: "|u1"}[dtype]
+        n = int(np.prod(shape)) * torch.empty((), dtype=dtype).element_size()
+        assert n <= self.nbytes
+
+        class _View:
+            __cuda_array_interface__ = {"shape": tuple(int(x) for x in shape), "typestr": typestr,
+                                        "data": (self.ptr, False), "version": 3}
+        t = torch.as_tensor(_View(), device="cuda")
+        return t.view(torch.bfloat16) if dtype == torch.bfloat16 else t
+
+    def trim(self, plan, guard_rows: int = 16) -> int:
+        freed = ctypes.c_int64()
+        _check(lib().dkv_vmm_trim(self, plan, int(guard_rows), ctypes.byref(freed)), "dkv_vmm_trim")
+        return freed.value
+
+    def mapped_bytes(self) -> int:
+        return int(lib().dkv_vmm_mapped_bytes(self))
+
+    def page_bytes(self) -> int:
+        return int(lib().dkv_vmm_page_bytes(self))
+
+    def close(self):
+        if self.handle:
+            lib().dkv_vmm_free(self)
+            self.handle = None
+
+
+def dkv_vmm_pages_to_keep(len_host, T_stride: int, reserve: int, guard_rows: int, page_bytes: int, npages: int,
+                          row_bytes: int = 256) -> np.ndarray:
+    ln = np.ascontiguousarray(len_host, np.int32)
+    keep = np.zeros(max(npages, 1), np.uint8)
+    lib().dkv_vmm_pages_to_keep(_ptr(ln), ln.size, int(T_stride), int(reserve), int(guard_rows), int(row_bytes),
+                                int(page_bytes), int(npages), _ptr(keep))
+    return keep[:npages]
 
 
 def dkv_plan_dense(ctx_len, shape: Shape, T_stride: int, stream=None) -> Plan:

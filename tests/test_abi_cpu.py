@@ -143,3 +143,32 @@ def test_topk_rejects_bad_arguments(dkvmod):
                                 (10, 3, fake, fake, ctypes.c_void_p(0x1002), ws_need)]:
         assert L.dkv_topk_mask(P, n, K, M, ws, wsb, None) == 1, (n, K)
         assert L.dkv_last_error()
+
+
+@pytest.mark.parametrize("page", [2 << 20, 65536, 1000])
+def test_vmm_page_rule_keeps_every_needed_row(dkvmod, page):
+    """dkv_vmm_pages_to_keep against an independent interval check: every byte a
+    slab may still touch (len + reserve + guard rows, capped at its region) is in
+    a kept page, and no page outside all of those is kept."""
+    rng = np.random.default_rng(page)
+    for trial in range(20):
+        NH = int(rng.integers(1, 40))
+        T = int(rng.integers(1, 20000))
+        reserve, guard = int(rng.integers(0, 300)), int(rng.integers(16, 64))
+        ln = rng.integers(0, T + 1, NH).astype(np.int32)
+        ln[rng.random(NH) < 0.2] = 0
+        total = NH * T * 256
+        npages = -(-total // page)
+        keep = dkvmod.dkv_vmm_pages_to_keep(ln, T, reserve, guard, page, npages)
+        want = np.zeros(npages, np.uint8)
+        for h in range(NH):
+            rows = min(T, int(ln[h]) + reserve + guard)
+            b0, b1 = h * T * 256, h * T * 256 + rows * 256
+            if rows > 0:
+                want[b0 // page:(b1 - 1) // page + 1] = 1
+        assert np.array_equal(keep, want), trial
+        for h in range(NH):  # the safety property itself
+            rows = min(T, int(ln[h]) + reserve + guard)
+            for b in (h * T * 256, h * T * 256 + rows * 256 - 1):
+                if rows > 0:
+                    assert keep[b // page] == 1
