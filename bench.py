@@ -272,35 +272,53 @@ def time_topk(wl, dev, reps=10):
 
 
 def time_compaction_inplace(wl, env, reps=5):
-    """dkv_compact_inplace on the dense caches (run last: it overwrites them).
-    Bytes: the rows that move (from the first dropped position of each slab on)
-    read and written, plus their indices."""
+    """The in-place path on page-backed caches: the dense K and V are copied into
+    dkv_vmm buffers, dkv_compact_inplace is timed there (median of reps; later
+    reps move already-moved bytes, the same volume), then dkv_vmm_trim releases
+    the pages no slab needs. Bytes: the rows that move (from the first dropped
+    position of each slab on), read and written, plus their indices."""
     import torch
 
     import paper_2609_32663_gb300.dkv as dkv
-    plan = dkv.dkv_map_pattern_inplace(env["M"], env["Tc"], env["shape"], env["T_stride"],
-                                       reserve_rows=env["reserve"])
+    T_stride, reserve = env["T_stride"], env["reserve"]
+    plan = dkv.dkv_map_pattern_inplace(env["M"], env["Tc"], env["shape"], T_stride, reserve_rows=reserve)
     ln, _, ioff, idx = dkv.dkv_plan_read(plan)
     moved = 0
     for h in range(len(ln)):
         ids = idx[ioff[h]:ioff[h + 1]]
         stay = np.flatnonzero(ids != np.arange(ids.size))
         moved += ids.size - (int(stay[0]) if stay.size else ids.size)
-    times = []
-    st = torch.cuda.current_stream()
-    for i in range(reps + 1):
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(st)
-        dkv.dkv_compact_inplace(plan, env["K"], env["V"])
-        e1.record(st)
-        e1.synchronize()
-        if i >= 1:
-            times.append(e0.elapsed_time(e1) * 1e-3)
-    plan.close()
+    shape = tuple(env["K"].shape)
+    nbytes = env["K"].numel() * 2
+    bufK, bufV = dkv.VmmBuffer(nbytes), dkv.VmmBuffer(nbytes)
+    try:
+        K, V = bufK.tensor(shape, torch.bfloat16), bufV.tensor(shape, torch.bfloat16)
+        K.copy_(env["K"])
+        V.copy_(env["V"])
+        times = []
+        st = torch.cuda.current_stream()
+        for i in range(reps + 1):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(st)
+            dkv.dkv_compact_inplace(plan, K, V)
+            e1.record(st)
+            e1.synchronize()
+            if i >= 1:
+                times.append(e0.elapsed_time(e1) * 1e-3)
+        mapped0 = bufK.mapped_bytes() + bufV.mapped_bytes()
+        freed = bufK.trim(plan, guard_rows=16) + bufV.trim(plan, guard_rows=16)
+        mapped1 = bufK.mapped_bytes() + bufV.mapped_bytes()
+        del K, V
+    finally:
+        plan.close()
+        bufK.close()
+        bufV.close()
     t = statistics.median(times)
     algo = moved * (2 * 256 * 2 + 4)
     return {"ms": round(t * 1e3, 3), "gbs": round(algo / t / 1e9, 1), "moved_rows": int(moved),
-            "kept_rows": int(ln.sum()), "how": "median of %d; later reps move already-moved bytes (same volume)" % reps}
+            "kept_rows": int(ln.sum()), "dense_bytes": int(mapped0), "mapped_after_trim": int(mapped1),
+            "freed_bytes": int(freed), "mapped_fraction": round(mapped1 / mapped0, 4),
+            "packed_bytes": int(ln.sum()) * 512, "how": "median of %d on dkv_vmm buffers, then dkv_vmm_trim" % reps}
 
 
 def time_multi_query(wl, env, dev, Q, steps, warmup):
