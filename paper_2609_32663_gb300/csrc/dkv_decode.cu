@@ -110,7 +110,8 @@ struct PK {
     static constexpr int kMetaBytes = NW * 6 * 4 + 16;  // first/last slab of each warp, their row bounds
     static constexpr int kFixedBytes = kRingBytes + kScratchBytes + kBarBytes + kMetaBytes;
     static constexpr int kStateFloats = G * (kHeadDim + 2);
-    static int bytes(int B) { return kFixedBytes + (2 * B + 1) * 4; }
+    static int bytes(int B) { return kFixedBytes + seq_table_bytes(B); }
+    static_assert(kFixedBytes + seq_table_bytes(kMaxB) <= 227 * 1024, "fits the opt-in shared memory of one CTA");
     static_assert(TR % RPS == 0 && 32 % TR == 0, "tile geometry");
     static_assert(kStateFloats * 4 <= NS * kStageBytes, "a warp's final state fits in its ring");
 };
@@ -323,9 +324,7 @@ __global__ void __launch_bounds__(C::NW * 32, 1) decode_partial_kernel(const Dec
     constexpr int G = C::G, LPR = C::LPR, TR = C::TR, NS = C::NS, NW = C::NW;
     constexpr int DPL = C::DPL, NCH = C::NCH, NSUM = C::NSUM;
     extern __shared__ __align__(128) unsigned char smem[];
-    SeqTable tab;
-    tab.NA = reinterpret_cast<int32_t*>(smem + C::kFixedBytes);
-    tab.NP = tab.NA + a.B;
+    const SeqTable tab = seq_table_at(smem + C::kFixedBytes, a);
     int32_t* seg_first = reinterpret_cast<int32_t*>(smem + C::kRingBytes + C::kScratchBytes + C::kBarBytes);
     int32_t* seg_last = seg_first + NW;
     int32_t* seg_p0 = seg_first + 2 * NW;  // [2 NW] layer rows [p0, p1) of entry 2 w (first) / 2 w + 1 (last)
@@ -337,7 +336,10 @@ __global__ void __launch_bounds__(C::NW * 32, 1) decode_partial_kernel(const Dec
     const int c = blockIdx.x;
     uint64_t* my_bars = reinterpret_cast<uint64_t*>(smem + C::kRingBytes + C::kScratchBytes) + warp * NS;
 
-    if (warp == 0) build_seq_table(a, tab, c == 0);
+    if (warp == 0)
+        build_seq_table(a, tab, c == 0);
+    else
+        load_slab_cache(a, tab, 32, (NW - 1) * 32);
     if (lane == 0) {
         for (int s = 0; s < NS; ++s) mbar_init(smem_u32(&my_bars[s]), 1);
         fence_proxy_async_smem();

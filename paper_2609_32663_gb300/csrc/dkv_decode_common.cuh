@@ -95,10 +95,48 @@ __device__ __forceinline__ void fence_proxy_async_smem()
 // Per-call sequence table in shared memory: NA[b] = rows already appended
 // (clamped to the reserve), NP[b] = exclusive prefix over b of the extra rows
 // e_b = NA[b] + (this call appends to b ? 1 : 0). Layer rows fit in int32.
+//
+// When the layer has fewer than kSlabCache slabs, the table also holds the
+// slabs' row prefix IO[h] = ioff[h] - ioff[0] ([NHl+1]) and cache offsets
+// OFF[h] = off[h] ([NHl]), so that finding a warp's rows and streaming them
+// reads no plan metadata from global memory: a CTA that starts after the
+// previous kernel has drained (the last ones to get an SM) would otherwise pay
+// a chain of dependent L2 round trips, under full HBM load, before its first
+// copy. IO and OFF are null for larger layers (read from global memory then).
+constexpr int kSlabCache = 1024;
 struct SeqTable {
-    int32_t* NA;  // [B]
-    int32_t* NP;  // [B+1]
+    int32_t* NA;   // [B]
+    int32_t* NP;   // [B+1]
+    int32_t* IO;   // [NHl+1] or null
+    int64_t* OFF;  // [NHl] or null
 };
+
+// Bytes of the table at an 8-byte aligned base: OFF, IO, NA, NP.
+__host__ __device__ constexpr int seq_table_bytes(int B) { return kSlabCache * 8 + kSlabCache * 4 + (2 * B + 1) * 4; }
+
+__device__ __forceinline__ SeqTable seq_table_at(unsigned char* base, const DecodeArgs& a)
+{
+    SeqTable t;
+    const bool cached = a.B * a.Hkv < kSlabCache;
+    t.OFF = cached ? reinterpret_cast<int64_t*>(base) : nullptr;
+    t.IO = cached ? reinterpret_cast<int32_t*>(base + kSlabCache * 8) : nullptr;
+    t.NA = reinterpret_cast<int32_t*>(base + kSlabCache * 12);
+    t.NP = t.NA + a.B;
+    return t;
+}
+
+// Fill IO and OFF (when cached) with the threads [t0, t0 + nt) of the CTA; the
+// caller's barrier publishes them.
+__device__ __forceinline__ void load_slab_cache(const DecodeArgs& a, SeqTable t, int t0, int nt)
+{
+    if (!t.IO) return;
+    const int NHl = a.B * a.Hkv;
+    const int64_t i0 = __ldg(a.ioff);
+    for (int h = (int)threadIdx.x - t0; h <= NHl; h += nt) {
+        t.IO[h] = (int)(__ldg(a.ioff + h) - i0);
+        if (h < NHl) t.OFF[h] = __ldg(a.off + h);
+    }
+}
 
 __device__ void build_seq_table(const DecodeArgs& a, SeqTable t, bool report)
 {
@@ -132,7 +170,7 @@ __device__ void build_seq_table(const DecodeArgs& a, SeqTable t, bool report)
 __device__ __forceinline__ int slab_start(const DecodeArgs& a, const SeqTable& t, int h)
 {
     const int b = h / a.Hkv, g = h - b * a.Hkv;
-    int p = (int)(a.ioff[h] - a.ioff[0]) + a.Hkv * t.NP[b];
+    int p = (t.IO ? t.IO[h] : (int)(a.ioff[h] - a.ioff[0])) + a.Hkv * t.NP[b];
     if (g) p += g * (t.NP[b + 1] - t.NP[b]);
     return p;
 }
@@ -202,9 +240,9 @@ __device__ __forceinline__ void cursor_seek(Cursor& cu, const DecodeArgs& a, con
         if (cu.s0 < cu.s1) {
             const int b = cu.h / a.Hkv;
             const int e = t.NP[b + 1] - t.NP[b];
-            cu.n_h = a.len[cu.h] + e;
+            cu.n_h = (t.IO ? t.IO[cu.h + 1] - t.IO[cu.h] : a.len[cu.h]) + e;
             cu.app = (a.append && e > t.NA[b]) ? 1 : 0;
-            cu.base = a.off[cu.h];
+            cu.base = t.OFF ? t.OFF[cu.h] : a.off[cu.h];
             cu.x = cu.s0;
             return;
         }

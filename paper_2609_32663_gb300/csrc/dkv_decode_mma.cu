@@ -45,7 +45,8 @@ struct MK {
     static constexpr int kMetaBytes = NW * 6 * 4 + 16;  // first/last slab of each warp, their row bounds
     static constexpr int kAlign = 1024;                  // swizzle atoms are 1024-byte aligned
     static constexpr int kFixedBytes = kRingBytes + kBarBytes + kMetaBytes;
-    static int bytes(int B) { return kAlign + kFixedBytes + (2 * B + 1) * 4; }
+    static int bytes(int B) { return kAlign + kFixedBytes + seq_table_bytes(B); }
+    static_assert(kAlign + kFixedBytes + seq_table_bytes(kMaxB) <= 227 * 1024, "fits the opt-in shared memory of one CTA");
     static_assert(8 * NT * (kHeadDim + 2) * 4 <= kWarpRing, "a warp's final state fits in its ring");
 };
 
@@ -338,9 +339,7 @@ __global__ void __launch_bounds__(MKFor<G, NT>::NW * 32, 1)
     extern __shared__ __align__(128) unsigned char smem_raw[];
     // The ring starts on a 1024-byte boundary (the swizzle pattern's period).
     unsigned char* smem = smem_raw + ((C::kAlign - (smem_u32(smem_raw) & (C::kAlign - 1))) & (C::kAlign - 1));
-    SeqTable tab;
-    tab.NA = reinterpret_cast<int32_t*>(smem + C::kFixedBytes);
-    tab.NP = tab.NA + a.B;
+    const SeqTable tab = seq_table_at(smem + C::kFixedBytes, a);
     int32_t* seg_first = reinterpret_cast<int32_t*>(smem + C::kRingBytes + C::kBarBytes);
     int32_t* seg_last = seg_first + NW;
     int32_t* seg_p0 = seg_first + 2 * NW;  // [2 NW] layer rows [p0, p1) of entry 2 w (first) / 2 w + 1 (last)
@@ -351,7 +350,10 @@ __global__ void __launch_bounds__(MKFor<G, NT>::NW * 32, 1)
     const int c = blockIdx.x;
     uint64_t* my_bars = reinterpret_cast<uint64_t*>(smem + C::kRingBytes) + warp * NS;
 
-    if (warp == 0) build_seq_table(a, tab, c == 0);
+    if (warp == 0)
+        build_seq_table(a, tab, c == 0);
+    else
+        load_slab_cache(a, tab, 32, (NW - 1) * 32);
     if (lane == 0) {
         for (int s = 0; s < NS; ++s) mbar_init(smem_u32(&my_bars[s]), 1);
         fence_proxy_async_smem();
