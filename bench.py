@@ -43,8 +43,8 @@ from paper_2609_32663_gb300 import inputs as I  # noqa: E402
 DECODE_TRAFFIC = {
     "sources": ("paper_2609_32663_gb300/csrc/dkv_decode_mma.cu", "paper_2609_32663_gb300/csrc/dkv_decode_common.cuh",
                 "paper_2609_32663_gb300/csrc/dkv_internal.cuh"),
-    "sha256": "f521f849ee27efecf3ee2e21335368568182c01b63da24a86f4fcc3537f35496",
-    "dram_bytes": 194_368_256 + 3_062_272,
+    "sha256": "4a31299690cbf9d19776186b16f999070fe0f31fede0ab14955ee7ac5341f88e",
+    "dram_bytes": 194_384_896 + 3_126_272,
     "algorithmic_bytes": 376_646 * 512 + 32 * 128 * (2 + 4),
     "capture": "profiles/decode_mma_llama8b-128k-l4.md",
 }
