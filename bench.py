@@ -42,8 +42,8 @@ from paper_2609_32663_gb300 import inputs as I  # noqa: E402
 # the value the capture was taken on (else the traffic is unknown: null).
 DECODE_TRAFFIC = {
     "sources": ("paper_2609_32663_gb300/csrc/dkv_decode_mma.cu", "paper_2609_32663_gb300/csrc/dkv_decode_common.cuh",
-                "paper_2609_32663_gb300/csrc/dkv_internal.cuh"),
-    "sha256": "4a31299690cbf9d19776186b16f999070fe0f31fede0ab14955ee7ac5341f88e",
+                "paper_2609_32663_gb300/csrc/dkv_ptx.cuh", "paper_2609_32663_gb300/csrc/dkv_internal.cuh"),
+    "sha256": "f20377960e7e51a9806a03cf0c5e11a8d51ab4e2d8a49a480dda0c7bf19f573b",
     "dram_bytes": 194_384_896 + 3_126_272,
     "algorithmic_bytes": 376_646 * 512 + 32 * 128 * (2 + 4),
     "capture": "profiles/decode_mma_llama8b-128k-l4.md",

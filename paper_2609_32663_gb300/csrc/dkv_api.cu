@@ -37,6 +37,7 @@ struct dkv_plan {
     int nctas_cap = 0, warps_cap = 0, cols_cap = 0;  // workspace sized for these
     int use_mma = 0;  // tensor-core decode kernel (needs the cache's row count for its tensor maps)
     int64_t inplace_stride = 0;  // > 0: slab h lives at rows h * stride of the dense buffer (in place)
+    int32_t* d_order = nullptr;  // in place: [NH] slabs by length, longest first, then a claim counter
 };
 
 namespace {
@@ -106,6 +107,7 @@ void release(dkv_plan* p)
     cudaFree(p->d_status);
     cudaFree(p->d_work);
     cudaFree(p->d_slab_count);
+    cudaFree(p->d_order);
     delete p;
 }
 
@@ -317,6 +319,25 @@ static dkv_status map_pattern_impl(const uint8_t* M_host, const int32_t* ctx_len
         return cuda_fail(e, "map: kernels");
     }
     cleanup();
+    if (inplace_stride > 0) {
+        // The in-place compaction streams whole slabs, longest first.
+        std::vector<int32_t> len((size_t)NH), order((size_t)NH + 1, 0);
+        if ((e = cudaMemcpy(len.data(), p->d_len, sizeof(int32_t) * NH, cudaMemcpyDeviceToHost)) != cudaSuccess) {
+            release(p);
+            return cuda_fail(e, "map: read lengths");
+        }
+        for (int h = 0; h < NH; ++h) order[(size_t)h] = h;
+        std::stable_sort(order.begin(), order.begin() + NH, [&](int32_t x, int32_t y) { return len[x] > len[y]; });
+        if ((st = dalloc(&p->d_order, (size_t)NH + 1, "slab order")) != DKV_OK) {
+            release(p);
+            return st;
+        }
+        if ((e = cudaMemcpy(p->d_order, order.data(), sizeof(int32_t) * (NH + 1), cudaMemcpyHostToDevice)) !=
+            cudaSuccess) {
+            release(p);
+            return cuda_fail(e, "map: slab order");
+        }
+    }
     if ((st = finish_plan(p)) != DKV_OK) {
         release(p);
         return st;
@@ -452,7 +473,8 @@ dkv_status dkv_compact_inplace(const dkv_plan* p, void* K, void* V, cudaStream_t
     a.T_stride = p->inplace_stride;
     a.kept = p->kept_rows;
     a.NH = p->s.L * p->B * p->s.H_kv;
-    dkv_status st = launched(dkv::launch_compact_inplace(a, stream), "in-place compact kernel");
+    dkv_status st =
+        launched(dkv::launch_compact_inplace(a, p->d_order, p->d_order + a.NH, stream), "in-place compact kernel");
     return st == DKV_OK ? ok() : st;
 }
 

@@ -83,68 +83,126 @@ __global__ void __launch_bounds__(kThreads) compact_kernel(const CompactArgs a)
 // In-place prune-and-pack: slab h's kept rows move from rows h * T_stride +
 // idx[r] to rows h * T_stride + r of the same buffer. idx is ascending, so
 // idx[r] >= r: a row only moves towards the slab's start, and rows before the
-// first dropped position stay where they are. One CTA walks a slab in chunks of
-// kInChunk rows: it loads the chunk's source rows into registers, waits at a
-// barrier for all of them, then stores. A chunk's sources lie at or after its
-// own destinations and strictly after the previous chunks' destinations, and
-// the next chunk's destinations come after this chunk's barrier, so no row is
-// overwritten before it has been read. Loads bypass L1 (the buffer is written
-// by this kernel).
-constexpr int kInThreads = 256;
-constexpr int kInChunk = 64;                               // rows per chunk
-constexpr int kInPer = kInChunk * 2 * 16 / kInThreads;     // 16-byte pieces per thread per chunk (K and V)
+// first dropped position stay where they are.
+//
+// One CTA per SM streams whole slabs, claimed from a list sorted by length
+// (longest first) so the last slabs to start are short. A slab's moving rows
+// go in chunks of kIpRows, in order: every thread loads its pieces of the
+// chunk's source rows into registers, a CTA barrier waits for all of them,
+// then the rows are stored at their destinations. A chunk's sources lie at or
+// after its own first destination and after every earlier chunk's
+// destinations, and the next chunk's stores come after this chunk's barrier,
+// so no row is overwritten before it has been read. The index entries of the
+// next chunk are loaded with this chunk's rows, off the critical path. Row
+// loads bypass L1 (the buffer is written by this kernel).
+namespace {
 
-__global__ void __launch_bounds__(kInThreads) compact_inplace_kernel(const CompactArgs a)
+constexpr int kIpThreads = 512;
+constexpr int kIpPer = 16;                               // 16-byte pieces per thread per chunk
+constexpr int kIpWarps = kIpThreads / 32;
+constexpr int kIpRows = kIpThreads * kIpPer / 32;        // rows per chunk (a row is 32 pieces: K, V)
+
+// Warp-wide search for the first row r in [0, n) with idx[r] > r (the predicate
+// is monotone: idx[r] - r is non-decreasing); n if none. Each round probes 32
+// evenly spaced rows, so a 64K-row slab takes four dependent loads.
+__device__ int first_moving_row(const int32_t* idx, int n, int lane)
 {
+    int lo = 0, hi = n;  // answer in [lo, hi]
+    while (hi - lo > 0) {
+        const int step = (hi - lo + 31) / 32;
+        const int x = lo + lane * step;
+        const bool p = x < hi && __ldg(idx + x) > x;
+        const unsigned m = __ballot_sync(0xffffffffu, p);
+        if (step == 1) return m ? lo + __ffs(m) - 1 : hi;
+        if (m) {
+            const int j = __ffs(m) - 1;  // x_j satisfies it, x_{j-1} does not
+            hi = lo + j * step;
+            lo = j ? lo + (j - 1) * step + 1 : lo;
+        } else {
+            lo += (hi - 1 - lo) / step * step + 1;  // past the last probed row
+        }
+    }
+    return lo;
+}
+
+__global__ void __launch_bounds__(kIpThreads, 1)
+    compact_inplace_kernel(const CompactArgs a, const int32_t* __restrict__ order, int32_t* claim)
+{
+    __shared__ int sh_h, sh_lo;
     uint16_t* K = const_cast<uint16_t*>(a.K);
     uint16_t* V = const_cast<uint16_t*>(a.V);
-    for (int h = blockIdx.x; h < a.NH; h += gridDim.x) {
-        const int n = a.len[h];
-        const int32_t* idx = a.idx + a.ioff[h];
-        const int64_t base = (int64_t)h * a.T_stride;
-        // First row that moves: idx[r] - r is non-decreasing, so a binary search.
-        int lo = 0, hi = n;
-        while (lo < hi) {
-            const int mid = (lo + hi) >> 1;
-            if (__ldg(idx + mid) > mid)
-                hi = mid;
-            else
-                lo = mid + 1;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int kv = (lane >> 4) & 1, c = lane & 15;  // a warp moves whole rows: K pieces, then V pieces
+    for (;;) {
+        __syncthreads();  // the previous slab's values of sh_h / sh_lo are no longer read
+        if (warp == 0) {
+            int h = -1, lo = 0;
+            int s = 0;
+            if (lane == 0) s = atomicAdd(claim, 1);
+            s = __shfl_sync(0xffffffffu, s, 0);
+            if (s < a.NH) {
+                h = __ldg(order + s);
+                lo = first_moving_row(a.idx + __ldg(a.ioff + h), __ldg(a.len + h), lane);
+            }
+            if (lane == 0) {
+                sh_h = h;
+                sh_lo = lo;
+            }
         }
-        for (int r0 = lo; r0 < n; r0 += kInChunk) {
-            uint4 v[kInPer];
-            int64_t dst[kInPer];
+        __syncthreads();
+        const int h = sh_h;
+        if (h < 0) return;
+        const int n = __ldg(a.len + h);
+        const int32_t* idx = a.idx + __ldg(a.ioff + h);
+        const int64_t base = (int64_t)h * a.T_stride;
+        int r0 = sh_lo;
+        // Piece i of this thread: row r0 + warp + kIpWarps * i of the chunk.
+        int nxt[kIpPer];
 #pragma unroll
-            for (int k = 0; k < kInPer; ++k) {
-                const int piece = threadIdx.x + k * kInThreads;  // (row, K/V, 16-byte chunk)
-                const int r = r0 + piece / 32, kv = (piece / 16) & 1, c = piece & 15;
-                dst[k] = -1;
-                if (r < n) {
-                    const uint16_t* src = (kv ? V : K) + (base + __ldg(idx + r)) * kHeadDim;
-                    v[k] = __ldcg(reinterpret_cast<const uint4*>(src) + c);
-                    dst[k] = ((base + r) * kHeadDim) / 8 + c;  // in uint4 units
+        for (int i = 0; i < kIpPer; ++i) {
+            const int r = r0 + warp + kIpWarps * i;
+            nxt[i] = r < n ? __ldg(idx + r) : -1;
+        }
+        for (; r0 < n; r0 += kIpRows) {
+            uint4 v[kIpPer];
+            int cur[kIpPer];
+#pragma unroll
+            for (int i = 0; i < kIpPer; ++i) {
+                cur[i] = nxt[i];
+                if (cur[i] >= 0) {
+                    const uint16_t* src = (kv ? V : K) + (base + cur[i]) * kHeadDim;
+                    v[i] = __ldcg(reinterpret_cast<const uint4*>(src) + c);
                 }
+            }
+#pragma unroll
+            for (int i = 0; i < kIpPer; ++i) {
+                const int r = r0 + kIpRows + warp + kIpWarps * i;
+                nxt[i] = r < n ? __ldg(idx + r) : -1;
             }
             __syncthreads();  // every source row of this chunk is read
 #pragma unroll
-            for (int k = 0; k < kInPer; ++k) {
-                const int piece = threadIdx.x + k * kInThreads;
-                const int kv = (piece / 16) & 1;
-                if (dst[k] >= 0) reinterpret_cast<uint4*>(kv ? V : K)[dst[k]] = v[k];
+            for (int i = 0; i < kIpPer; ++i) {
+                if (cur[i] >= 0) {
+                    const int64_t dst = base + r0 + warp + kIpWarps * i;
+                    reinterpret_cast<uint4*>((kv ? V : K) + dst * kHeadDim)[c] = v[i];
+                }
             }
         }
     }
 }
 
-cudaError_t launch_compact_inplace(const CompactArgs& a, cudaStream_t st)
+}  // namespace
+
+cudaError_t launch_compact_inplace(const CompactArgs& a, const int32_t* order, int32_t* claim, cudaStream_t st)
 {
     if (a.kept == 0 || a.NH == 0) return cudaSuccess;
     int dev = 0, sms = 0;
     cudaError_t e;
     if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
     if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-    const int grid = a.NH < 8 * sms ? a.NH : 8 * sms;
-    compact_inplace_kernel<<<grid, kInThreads, 0, st>>>(a);
+    if ((e = cudaMemsetAsync(claim, 0, sizeof(int32_t), st)) != cudaSuccess) return e;
+    const int grid = a.NH < sms ? a.NH : sms;
+    compact_inplace_kernel<<<grid, kIpThreads, 0, st>>>(a, order, claim);
     return cudaGetLastError();
 }
 

@@ -49,7 +49,8 @@ struct CompactArgs {
 cudaError_t launch_compact(const CompactArgs& a, cudaStream_t st);
 // In place: K and V are both source and destination, slab h at rows h * T_stride
 // (Kc/Vc unused); every slab's kept rows move to its first len rows, in order.
-cudaError_t launch_compact_inplace(const CompactArgs& a, cudaStream_t st);
+// order: the NH slabs, longest first; claim: a counter the launch zeroes.
+cudaError_t launch_compact_inplace(const CompactArgs& a, const int32_t* order, int32_t* claim, cudaStream_t st);
 
 // ---------------------------------------------------------------- decode
 struct DecodeArgs {

@@ -98,6 +98,13 @@ def test_inplace_all_drop_and_short_contexts(cuda):
     run(w, reserve=2, M=M, Tc=Tc, steps=2, cuda=cuda)
 
 
+def test_inplace_many_short_slabs(cuda):
+    """More slabs than SMs, most of them short: the kernel's CTAs claim slabs
+    one after another, and slabs where no row moves are skipped."""
+    w = wl(L=4, H=8, Hkv=4, B=16, T=3000, D=20, W=-(-(3000 - 1152) // 20), ragged=(0, 3000), seed=54)
+    run(w, reserve=2, steps=1, cuda=cuda)
+
+
 def test_inplace_rejects_short_stride_and_wrong_plan(cuda):
     w = wl(seed=53)
     sh, _ = shapes(w)
