@@ -336,14 +336,17 @@ void dkv_free(dkv_plan* plan);
  *                (host only). Returns -1 when rho is outside [0, 1] or a size is
  *                negative.
  * dkv_topk_workspace_bytes
- *                device workspace bytes dkv_topk_mask needs (a few KB, the same
- *                for every n).
+ *                device workspace bytes dkv_topk_mask needs (about 29 KB, the
+ *                same for every n).
  * dkv_topk_mask  P: device float [n], any layout, read in flat order.
  *                M: device uint8 [n], written in full. M[i] = 1 for the K first
  *                entries in this order: larger value first; equal values (+0
  *                and -0 are equal) by lower flat index; NaN after every number.
  *                workspace: device scratch of at least dkv_topk_workspace_bytes()
  *                bytes, 4-byte aligned; calls that share it must be ordered.
+ *                Its first 32-bit word is a status word: nonzero after a call
+ *                whose grid barrier wait ran out (M is then incomplete).
+ *                One cooperative launch (all its CTAs resident at once).
  *                Asynchronous on stream; allocates nothing.
  * Errors: DKV_ERR_INVALID_ARG (n < 0 or n >= 2^31, K outside [0, n], a NULL
  * pointer with n > 0, a small or unaligned workspace), DKV_ERR_CUDA.

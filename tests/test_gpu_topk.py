@@ -24,8 +24,11 @@ def gpu_mask(P, K, cuda):
     Pd = torch.from_numpy(np.ascontiguousarray(P, np.float32)).to(cuda)
     Md = torch.full(Pd.shape, 7, dtype=torch.uint8, device=cuda)  # every byte must be written
     ws = torch.empty(dkv.dkv_topk_workspace_bytes() // 4 + 1, dtype=torch.int32, device=cuda)
+    ws[0] = 0
     dkv.dkv_topk_mask(Pd, K, Md, ws)
     torch.cuda.synchronize()
+    if 0 < K < P.size:
+        assert int(ws[0].item()) == 0  # no grid barrier wait ran out
     return Md.cpu().numpy()
 
 
