@@ -131,6 +131,17 @@ def test_decode_many_sequences_uneven():
     c.close()
 
 
+@pytest.mark.parametrize("G", [4, 7])
+def test_decode_more_slabs_than_the_shared_table(G):
+    """B * H_kv >= 1024 slabs in a layer: the kernels read slab starts and cache
+    offsets from global memory instead of their shared-memory copy."""
+    w = wl(L=1, H=8 * G, Hkv=8, T=1300, B=130, D=2, W=(1300 - 1152) // 2, ragged=(0, 1300), seed=80 + G)
+    assert w.B * w.Hkv >= 1024
+    c = Case(w, reserve=2)
+    c.decode_steps(1, append=True)
+    c.close()
+
+
 def test_decode_outlier_keys_and_custom_scale():
     w = wl(H=8, Hkv=2, T=9000, D=8, W=(9000 - 1152) // 8, outlier_frac=0.05, seed=5)
     c = Case(w)
