@@ -368,6 +368,22 @@ def time_multi_query(wl, env, dev, Q, steps, warmup):
     return e0.elapsed_time(e1) * 1e-3 / steps
 
 
+def profile_multi_query(wl, env, dev, Qs=(2, 4)):
+    """Eager dkv_decode_multi launches, one per layer for each Q, untimed: the
+    timed multi-query runs are graph replays, and these are the launches a
+    profiler selects."""
+    import torch
+
+    import paper_2609_32663_gb300.dkv as dkv
+    n_app = torch.zeros(wl.B, dtype=torch.int32, device=dev)
+    for Q in Qs:
+        q = torch.randn((wl.B, Q, wl.H, wl.head_dim), device=dev).to(torch.bfloat16)
+        out = torch.empty((wl.B, Q, wl.H, wl.head_dim), dtype=torch.float32, device=dev)
+        for layer in range(wl.L):
+            dkv.dkv_decode_multi(env["plan"], layer, q, Q, n_app, env["Kc"], env["Vc"], out)
+    torch.cuda.synchronize()
+
+
 def step_bytes(wl, Tc_rows_per_layer, with_new=True):
     """Algorithmic bytes of one decode step: retained K/V rows (with appended
     tokens) + q read + o written + the new K/V row written."""
@@ -580,6 +596,8 @@ def run_dkv(args, dist):
     n_inst = 4 if args.profile else 16
     before = runner.n_app.clone()
     t_part, n_launch = runner.timed_launches(n_inst)
+    if args.profile:
+        profile_multi_query(wl, env, dev)
     napp_inst = float(before[0].item()) + (n_inst - 1) / 2.0
     rows_launch = (sum(rows_layer) + wl.L * NHl * (napp_inst + 1)) / wl.L
     part_bytes = rows_launch * 512 + wl.B * wl.H * (256 + 512) + 4 * wl.B * wl.Hkv * 256
