@@ -54,7 +54,8 @@ def run_case(w, Q, steps_before=2):
     case.close()
 
 
-@pytest.mark.parametrize("G,Q", [(4, 1), (4, 2), (4, 3), (4, 4), (7, 1), (7, 2), (8, 2), (1, 8), (1, 16), (2, 5)])
+@pytest.mark.parametrize("G,Q", [(4, 1), (4, 2), (4, 3), (4, 4), (7, 1), (7, 2), (8, 2), (1, 8), (1, 16), (2, 5),
+                                 (3, 5), (5, 3), (6, 2), (2, 8)])
 def test_multi_query_matches_oracle(G, Q):
     run_case(wl(H=2 * G, Hkv=2, seed=G * 10 + Q), Q)
 

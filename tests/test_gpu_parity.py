@@ -93,14 +93,14 @@ def test_compact_bytes_match_oracle(G, B, reserve):
 
 # ---------------------------------------------------------------- decode (tolerance)
 
-@pytest.mark.parametrize("G", [1, 4, 7, 8])
+@pytest.mark.parametrize("G", [1, 2, 3, 4, 5, 6, 7, 8])
 def test_decode_matches_oracle_without_append(G):
     c = Case(wl(H=2 * G, Hkv=2, T=6000, B=2, D=8, W=606, ragged=(1000, 6000), seed=20 + G))
     c.decode_steps(1, append=False)
     c.close()
 
 
-@pytest.mark.parametrize("G", [1, 4, 7])
+@pytest.mark.parametrize("G", [1, 3, 4, 5, 6, 7])
 def test_decode_with_appends_over_steps(G):
     c = Case(wl(H=2 * G, Hkv=2, T=5000, B=3, D=8, W=500, ragged=(100, 5000), seed=30 + G), reserve=6)
     c.decode_steps(4, append=True)
