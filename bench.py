@@ -19,6 +19,7 @@ its own replica (the path does not exchange data between GPUs); the timing is
 the max over ranks and rank 0 prints one JSON line.
 """
 import argparse
+import contextlib
 import json
 import os
 import statistics
@@ -68,6 +69,17 @@ UNIT = "us/step"
 
 DEFAULT_STEPS = 256
 DEFAULT_WARMUP = 8
+
+
+@contextlib.contextmanager
+def nvtx(name):
+    """An NVTX range around a bench phase (visible to a timeline profiler)."""
+    import torch
+    torch.cuda.nvtx.range_push(name)
+    try:
+        yield
+    finally:
+        torch.cuda.nvtx.range_pop()
 
 
 def reserve_rows(steps, warmup):
@@ -574,8 +586,10 @@ def run_dkv(args, dist):
     if args.profile:
         steps, warmup = min(steps, 2), min(warmup, 3)
     reserve = reserve_rows(steps, warmup)
-    env = setup(wl, dev, reserve)
-    comp = time_compaction(env, reps=3 if args.profile else 10)
+    with nvtx("setup: map, dense caches"):
+        env = setup(wl, dev, reserve)
+    with nvtx("compaction"):
+        comp = time_compaction(env, reps=3 if args.profile else 10)
     info = env["info"]
     NHl = wl.B * wl.Hkv
     ln, *_ = dkv.dkv_plan_read(env["plan"])
@@ -584,7 +598,8 @@ def run_dkv(args, dist):
     runner = DecodeRunner(wl, env["plan"], env["Kc"], env["Vc"], dev)
     runner.capture()
     clocks = Clocks(dist.local)
-    t_step, clk = time_graph(runner, steps, warmup, dist, clocks)
+    with nvtx("decode step graph (timed)"):
+        t_step, clk = time_graph(runner, steps, warmup, dist, clocks)
     t_step = dist.max(t_step)
     # Rows attended per step (the cache grows by one row per slab per step).
     napp_mid = warmup + (steps - 1) / 2.0
@@ -595,9 +610,11 @@ def run_dkv(args, dist):
     # launch (one layer): retained K/V rows + q read + o written + new K/V row in and out.
     n_inst = 4 if args.profile else 16
     before = runner.n_app.clone()
-    t_part, n_launch = runner.timed_launches(n_inst)
+    with nvtx("decode launches (eager, timed)"):
+        t_part, n_launch = runner.timed_launches(n_inst)
     if args.profile:
-        profile_multi_query(wl, env, dev)
+        with nvtx("multi-query launches (eager)"):
+            profile_multi_query(wl, env, dev)
     napp_inst = float(before[0].item()) + (n_inst - 1) / 2.0
     rows_launch = (sum(rows_layer) + wl.L * NHl * (napp_inst + 1)) / wl.L
     part_bytes = rows_launch * 512 + wl.B * wl.H * (256 + 512) + 4 * wl.B * wl.Hkv * 256
@@ -649,7 +666,8 @@ def run_dkv(args, dist):
         dense = dkv.dkv_plan_dense(env["Tc"], env["shape"], T_stride=env["T_stride"])
         dr = DecodeRunner(wl, dense, env["K"], env["V"], dev)
         dr.capture()
-        t_dense, _ = time_graph(dr, steps, warmup, dist)
+        with nvtx("dense baseline graph (timed)"):
+            t_dense, _ = time_graph(dr, steps, warmup, dist)
         t_dense = dist.max(t_dense)
         dense_rows = wl.L * float(env["Tc"].sum()) * wl.Hkv + wl.L * NHl * (napp_mid + 1)
         res["dense_baseline"] = {"us_per_step": round(t_dense * 1e6, 2),
@@ -661,7 +679,8 @@ def run_dkv(args, dist):
 
     # End to end through the public API with host buffers (fresh plan state).
     env2_plan = env["plan"]
-    t_e2e, bi, bo = run_e2e(wl, env2_plan, env["Kc"], env["Vc"], dev, max(8, min(steps, 32)), warmup)
+    with nvtx("e2e graph with host copies (timed)"):
+        t_e2e, bi, bo = run_e2e(wl, env2_plan, env["Kc"], env["Vc"], dev, max(8, min(steps, 32)), warmup)
     t_e2e = dist.max(t_e2e)
     res["e2e"] = {"value": round(t_e2e * 1e6, 2), "unit": UNIT, "h2d_bytes_per_step": int(bi),
                   "d2h_bytes_per_step": int(bo), "steps": max(8, min(steps, 32)),
@@ -670,22 +689,26 @@ def run_dkv(args, dist):
 
     if dist.rank == 0 and dist.world == 1 and not args.no_cpu and not args.profile:
         layers = max(1, min(args.cpu_layers, wl.L))
-        t_cpu, rows = cpu_oracle_step(wl, env, layers, dev)
+        with nvtx("CPU oracle"):
+            t_cpu, rows = cpu_oracle_step(wl, env, layers, dev)
         res["cpu_baseline"] = {"value": round(t_cpu * 1e6, 1), "unit": UNIT, "cores": 1, "kind": "oracle",
                                "sample": f"fp64 scalar oracle, {layers} of {wl.L} layers of one decode step "
                                          f"({rows} rows x G={wl.G} heads), scaled x{wl.L / layers:g} to a step",
                                "cpu": cpu_model(), "nproc": os.cpu_count()}
     if not args.profile:
-        res["pattern_export"] = time_topk(wl, dev)
+        with nvtx("pattern export"):
+            res["pattern_export"] = time_topk(wl, dev)
         mq = {}
         for Q in sorted({1, max(1, 8 // wl.G), max(1, 16 // wl.G)}):
-            t_q = dist.max(time_multi_query(wl, env, dev, Q, min(steps, 64), warmup))
+            with nvtx(f"multi-query Q={Q} graph (timed)"):
+                t_q = dist.max(time_multi_query(wl, env, dev, Q, min(steps, 64), warmup))
             rows_q = sum(rows_layer)  # no appends in these calls
             mq[f"Q{Q}"] = {"us_per_step": round(t_q * 1e6, 2), "queries_per_s": round(wl.B * Q * dist.world / t_q, 1),
                            "gbs": round(step_bytes(wl, rows_q, with_new=False) / t_q / 1e9, 1)}
         res["multi_query"] = mq
     if not args.profile:
-        res["compaction_inplace"] = time_compaction_inplace(wl, env)  # last: overwrites the dense caches
+        with nvtx("in-place compaction"):
+            res["compaction_inplace"] = time_compaction_inplace(wl, env)  # last: overwrites the dense caches
     st = dkv.dkv_plan_status(env["plan"])
     res["device_status_word"] = st
     env["plan"].close()
