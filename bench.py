@@ -44,7 +44,7 @@ from paper_2609_32663_gb300 import inputs as I  # noqa: E402
 DECODE_TRAFFIC = {
     "sources": ("paper_2609_32663_gb300/csrc/dkv_decode_mma.cu", "paper_2609_32663_gb300/csrc/dkv_decode_common.cuh",
                 "paper_2609_32663_gb300/csrc/dkv_ptx.cuh", "paper_2609_32663_gb300/csrc/dkv_internal.cuh"),
-    "sha256": "f20377960e7e51a9806a03cf0c5e11a8d51ab4e2d8a49a480dda0c7bf19f573b",
+    "sha256": "e260ff53f18b4659dba991023e92c78792286a3bc7c9fac6c4e2216ff590691a",
     "dram_bytes": 194_384_896 + 3_126_272,
     "algorithmic_bytes": 376_646 * 512 + 32 * 128 * (2 + 4),
     "capture": "profiles/decode_mma_llama8b-128k-l4.md",

@@ -29,7 +29,7 @@
 namespace dkv {
 namespace {
 
-// (constants, PTX helpers, partition and merge helpers: dkv_decode_common.cuh)
+// (constants, partition and merge helpers: dkv_decode_common.cuh; PTX wrappers: dkv_ptx.cuh)
 
 // ------------------------------------------------------------ partial kernel
 // Packed pair of fp32 values (one 64-bit register pair) for fma.rn.f32x2.

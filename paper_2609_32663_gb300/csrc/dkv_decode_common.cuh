@@ -1,6 +1,6 @@
 // Pieces shared by the decode kernels (split-K over the packed cache, Sec. 3.4):
-// PTX wrappers (mbarrier, bulk copies, programmatic dependent launch), the
-// stream-K row partition over the slabs of one layer, the tile cursor of a
+// programmatic-dependent-launch wrappers (the mbarrier and bulk-copy ones are in
+// dkv_ptx.cuh), the per-call slab table, the stream-K row partition over the slabs of one layer, the tile cursor of a
 // warp, and the end of a CTA's pass: merging the warp states that share a slab
 // and the fused cross-CTA merge (the last CTA to finish a (slab, head) merges
 // every CTA's partial of it).
