@@ -148,6 +148,44 @@ def _ptr(t):
     return t.data_ptr()
 
 
+def _dev(t, name, dtypes=None, numel=None, min_numel=None):
+    """Address of a device buffer argument, checked: a contiguous CUDA tensor of
+    the expected element type and size (an int is taken as a raw device address,
+    None as NULL). A host tensor passed here would make the kernel read host
+    addresses, so it is refused before the call."""
+    if t is None or isinstance(t, int):
+        return t
+    why = None
+    if not getattr(t, "is_cuda", False):
+        why = "must be a CUDA tensor"
+    elif not t.is_contiguous():
+        why = "must be contiguous"
+    elif dtypes is not None and t.dtype not in dtypes:
+        why = f"has dtype {t.dtype}, expected one of {dtypes}"
+    elif numel is not None and t.numel() != numel:
+        why = f"has {t.numel()} elements, expected {numel}"
+    elif min_numel is not None and t.numel() < min_numel:
+        why = f"has {t.numel()} elements, needs at least {min_numel}"
+    if why:
+        raise DkvError(DKV_ERR_INVALID_ARG, "argument check", f"{name} {why}")
+    return t.data_ptr()
+
+
+def _bf16():
+    import torch
+    return (torch.bfloat16, torch.int16)
+
+
+def _i32():
+    import torch
+    return (torch.int32,)
+
+
+def _f32():
+    import torch
+    return (torch.float32,)
+
+
 def _stream(stream):
     if stream is None:
         import torch
@@ -207,7 +245,9 @@ def dkv_map_pattern_inplace(M, ctx_len, shape: Shape, T_stride: int, reserve_row
 
 def dkv_compact_inplace(plan: Plan, K, V, stream=None):
     """Move each slab's kept rows to the start of its region of K and V (in place)."""
-    _check(lib().dkv_compact_inplace(plan, _ptr(K), _ptr(V), _stream(stream)), "dkv_compact_inplace")
+    need = dkv_plan_query(plan).total_rows * 128
+    _check(lib().dkv_compact_inplace(plan, _dev(K, "K", _bf16(), min_numel=need), _dev(V, "V", _bf16(), min_numel=need),
+                                     _stream(stream)), "dkv_compact_inplace")
 
 
 class VmmBuffer:
@@ -290,39 +330,60 @@ def dkv_plan_query(plan: Plan) -> PlanInfo:
 def dkv_compact(plan: Plan, K, V, Kc, Vc, T_stride: int | None = None, stream=None):
     if T_stride is None:
         T_stride = K.shape[-2]
-    _check(lib().dkv_compact(plan, _ptr(K), _ptr(V), int(T_stride), _ptr(Kc), _ptr(Vc), _stream(stream)),
-           "dkv_compact")
+    sh = plan.shape
+    dense = sh.L * plan.B * sh.H_kv * int(T_stride) * 128
+    packed = dkv_plan_query(plan).total_rows * 128
+    _check(lib().dkv_compact(plan, _dev(K, "K", _bf16(), min_numel=dense), _dev(V, "V", _bf16(), min_numel=dense),
+                             int(T_stride), _dev(Kc, "Kc", _bf16(), min_numel=packed),
+                             _dev(Vc, "Vc", _bf16(), min_numel=packed), _stream(stream)), "dkv_compact")
+
+
+def _decode_ptrs(plan: Plan, q, k_new, v_new, n_appended, Kc, Vc, Q: int = 1):
+    sh, B = plan.shape, plan.B
+    rows = dkv_plan_query(plan).total_rows * 128
+    return (_dev(q, "q", _bf16(), numel=B * Q * sh.H * 128),
+            _dev(k_new, "k_new", _bf16(), numel=B * sh.H_kv * 128),
+            _dev(v_new, "v_new", _bf16(), numel=B * sh.H_kv * 128),
+            _dev(n_appended, "n_appended", _i32(), numel=B),
+            _dev(Kc, "Kc", _bf16(), min_numel=rows), _dev(Vc, "Vc", _bf16(), min_numel=rows))
 
 
 def dkv_decode_attn(plan: Plan, layer: int, q, k_new, v_new, n_appended, Kc, Vc, out, scale: float = 0.0,
                     stream=None):
-    _check(lib().dkv_decode_attn(plan, int(layer), _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(n_appended),
-                                 _ptr(Kc), _ptr(Vc), ctypes.c_float(scale), _ptr(out), _stream(stream)),
-           "dkv_decode_attn")
+    qp, kp, vp, np_, kc, vc = _decode_ptrs(plan, q, k_new, v_new, n_appended, Kc, Vc)
+    op = _dev(out, "out", _f32(), numel=plan.B * plan.shape.H * 128)
+    _check(lib().dkv_decode_attn(plan, int(layer), qp, kp, vp, np_, kc, vc, ctypes.c_float(scale), op,
+                                 _stream(stream)), "dkv_decode_attn")
 
 
 def dkv_decode_multi(plan: Plan, layer: int, q, num_queries: int, n_appended, Kc, Vc, out, scale: float = 0.0,
                      stream=None):
     """num_queries queries per sequence over the same compressed rows: q bf16
     [B][Q][H][128] -> out fp32 [B][Q][H][128]."""
-    _check(lib().dkv_decode_multi(plan, int(layer), _ptr(q), int(num_queries), _ptr(n_appended), _ptr(Kc), _ptr(Vc),
-                                  ctypes.c_float(scale), _ptr(out), _stream(stream)), "dkv_decode_multi")
+    Q = max(int(num_queries), 1)
+    qp, _, _, np_, kc, vc = _decode_ptrs(plan, q, None, None, n_appended, Kc, Vc, Q=Q)
+    op = _dev(out, "out", _f32(), numel=plan.B * Q * plan.shape.H * 128)
+    _check(lib().dkv_decode_multi(plan, int(layer), qp, int(num_queries), np_, kc, vc, ctypes.c_float(scale), op,
+                                  _stream(stream)), "dkv_decode_multi")
 
 
 def dkv_decode_partial(plan: Plan, layer: int, q, k_new, v_new, n_appended, Kc, Vc, scale: float = 0.0,
                        stream=None):
-    _check(lib().dkv_decode_partial(plan, int(layer), _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(n_appended),
-                                    _ptr(Kc), _ptr(Vc), ctypes.c_float(scale), _stream(stream)),
-           "dkv_decode_partial")
+    qp, kp, vp, np_, kc, vc = _decode_ptrs(plan, q, k_new, v_new, n_appended, Kc, Vc)
+    _check(lib().dkv_decode_partial(plan, int(layer), qp, kp, vp, np_, kc, vc, ctypes.c_float(scale),
+                                    _stream(stream)), "dkv_decode_partial")
 
 
 def dkv_decode_combine(plan: Plan, layer: int, n_appended, with_new_token: bool, out, stream=None):
-    _check(lib().dkv_decode_combine(plan, int(layer), _ptr(n_appended), int(bool(with_new_token)), _ptr(out),
-                                    _stream(stream)), "dkv_decode_combine")
+    np_ = _dev(n_appended, "n_appended", _i32(), numel=plan.B)
+    op = _dev(out, "out", _f32(), numel=plan.B * plan.shape.H * 128)
+    _check(lib().dkv_decode_combine(plan, int(layer), np_, int(bool(with_new_token)), op, _stream(stream)),
+           "dkv_decode_combine")
 
 
 def dkv_advance(plan: Plan, n_appended, stream=None):
-    _check(lib().dkv_advance(plan, _ptr(n_appended), _stream(stream)), "dkv_advance")
+    _check(lib().dkv_advance(plan, _dev(n_appended, "n_appended", _i32(), numel=plan.B), _stream(stream)),
+           "dkv_advance")
 
 
 def dkv_plan_status(plan: Plan, clear: bool = False, stream=None) -> int:
@@ -349,12 +410,13 @@ def dkv_topk_workspace_bytes() -> int:
 
 def dkv_topk_mask(P, K: int, M, workspace, stream=None):
     """M (device uint8, same element count as P) = TopKMask(P, K) of Eq. 3."""
+    import torch
     n = P.numel()
-    if M.numel() != n:
-        raise ValueError("M must have as many elements as P")
+    pp = _dev(P, "P", _f32())
+    mp = _dev(M, "M", (torch.uint8,), numel=n)
+    wp = _dev(workspace, "workspace")
     nbytes = workspace.numel() * workspace.element_size()
-    _check(lib().dkv_topk_mask(_ptr(P), int(n), int(K), _ptr(M), _ptr(workspace), int(nbytes), _stream(stream)),
-           "dkv_topk_mask")
+    _check(lib().dkv_topk_mask(pp, int(n), int(K), mp, wp, int(nbytes), _stream(stream)), "dkv_topk_mask")
 
 
 def dkv_decode_attn_noalloc(shape: Shape, B: int, layer: int, reserve_rows: int, d_len, d_off, d_ioff, q, k_new,
@@ -362,11 +424,13 @@ def dkv_decode_attn_noalloc(shape: Shape, B: int, layer: int, reserve_rows: int,
     """Decode attention that allocates no device memory; d_len/d_off/d_ioff are
     device addresses (ints) or tensors of the plan metadata."""
     sh = shape.c()
-    addr = (lambda t: t if isinstance(t, int) or t is None else _ptr(t))
-    _check(lib().dkv_decode_attn_noalloc(ctypes.byref(sh), int(B), int(layer), int(reserve_rows), addr(d_len),
-                                         addr(d_off), addr(d_ioff), _ptr(q), _ptr(k_new), _ptr(v_new),
-                                         _ptr(n_appended), _ptr(Kc), _ptr(Vc), ctypes.c_float(scale), _ptr(out),
-                                         _ptr(status), _stream(stream)), "dkv_decode_attn_noalloc")
+    _check(lib().dkv_decode_attn_noalloc(
+        ctypes.byref(sh), int(B), int(layer), int(reserve_rows), _dev(d_len, "d_len"), _dev(d_off, "d_off"),
+        _dev(d_ioff, "d_ioff"), _dev(q, "q", _bf16(), numel=B * shape.H * 128),
+        _dev(k_new, "k_new", _bf16(), numel=B * shape.H_kv * 128), _dev(v_new, "v_new", _bf16(), numel=B * shape.H_kv * 128),
+        _dev(n_appended, "n_appended", _i32(), numel=B), _dev(Kc, "Kc", _bf16()), _dev(Vc, "Vc", _bf16()),
+        ctypes.c_float(scale), _dev(out, "out", _f32(), numel=B * shape.H * 128), _dev(status, "status", _i32()),
+        _stream(stream)), "dkv_decode_attn_noalloc")
 
 
 def dkv_plan_read(plan: Plan, stream=None):

@@ -290,3 +290,29 @@ def test_unaligned_pointer_rejected():
     with pytest.raises(dkv.DkvError):
         dkv.dkv_decode_attn(c.plan, 2, q, None, None, None, c.Kc, c.Vc, out)  # layer out of range
     c.close()
+
+
+def test_binding_refuses_host_and_mistyped_buffers(cuda):
+    """The Python binding checks device-buffer arguments before the call: a host
+    tensor, a wrong element type or a short cache is refused with
+    DKV_ERR_INVALID_ARG (a host address reaching a kernel would fault)."""
+    c = Case(wl(seed=9))
+    w = c.wl
+    q = torch.zeros((w.B, w.H, 128), dtype=torch.bfloat16, device=c.dev)
+    out = torch.empty((w.B, w.H, 128), dtype=torch.float32, device=c.dev)
+    bad = [
+        dict(q=q.cpu()),
+        dict(q=q.float()),
+        dict(out=out.to(torch.bfloat16)),
+        dict(out=torch.empty((w.B, w.H + 1, 128), dtype=torch.float32, device=c.dev)),
+        dict(Kc=c.Kc[:-1]),
+    ]
+    for b in bad:
+        args = dict(q=q, Kc=c.Kc, Vc=c.Vc, out=out)
+        args.update(b)
+        with pytest.raises(dkv.DkvError) as e:
+            dkv.dkv_decode_attn(c.plan, 0, args["q"], None, None, None, args["Kc"], args["Vc"], args["out"])
+        assert e.value.status == dkv.DKV_ERR_INVALID_ARG
+    dkv.dkv_decode_attn(c.plan, 0, q, None, None, None, c.Kc, c.Vc, out)  # the valid call still runs
+    torch.cuda.synchronize()
+    c.close()
