@@ -316,3 +316,18 @@ def test_binding_refuses_host_and_mistyped_buffers(cuda):
     dkv.dkv_decode_attn(c.plan, 0, q, None, None, None, c.Kc, c.Vc, out)  # the valid call still runs
     torch.cuda.synchronize()
     c.close()
+
+
+def test_decode_at_the_batch_limit():
+    """B = 512 sequences (the kernels' per-call table limit), one KV head each."""
+    w = wl(L=1, H=4, Hkv=1, T=1300, B=512, D=2, W=(1300 - 1152) // 2, ragged=(0, 1300), seed=88)
+    c = Case(w, reserve=1)
+    c.decode_steps(1, append=True)
+    c.close()
+
+
+def test_batch_above_the_limit_is_refused():
+    w = wl(L=1, H=4, Hkv=1, T=64, B=513, D=2, W=64, seed=89)
+    sh, _ = shapes(w)
+    with pytest.raises(dkv.DkvError):
+        dkv.dkv_map_pattern(I.make_pattern(w), I.context_lengths(w), sh, reserve_rows=0)
