@@ -44,7 +44,7 @@ from paper_2609_32663_gb300 import inputs as I  # noqa: E402
 DECODE_TRAFFIC = {
     "sources": ("paper_2609_32663_gb300/csrc/dkv_decode_mma.cu", "paper_2609_32663_gb300/csrc/dkv_decode_common.cuh",
                 "paper_2609_32663_gb300/csrc/dkv_ptx.cuh", "paper_2609_32663_gb300/csrc/dkv_internal.cuh"),
-    "sha256": "e260ff53f18b4659dba991023e92c78792286a3bc7c9fac6c4e2216ff590691a",
+    "sha256": "ebf061ffdaf63866f9922d4a34ae06a46572ad5c54a34cd993e091e9956df50e",
     "dram_bytes": 194_384_896 + 3_126_272,
     "algorithmic_bytes": 376_646 * 512 + 32 * 128 * (2 + 4),
     "capture": "profiles/decode_mma_llama8b-128k-l4.md",
