@@ -78,6 +78,17 @@ def test_tiny_and_ragged_sizes(cuda):
             assert np.array_equal(gpu_mask(P, K, cuda), O.topk_mask(P, K)), (n, K)
 
 
+@pytest.mark.parametrize("n", [393_215, 400_000, 1_000_003])
+def test_special_values_on_many_ctas(n, cuda):
+    """Ties, NaN, +-0 and +-inf spread over many CTAs of the grid (the tie
+    prefix crosses CTA and warp ranges)."""
+    rng = np.random.default_rng(n)
+    vals = np.array([0.0, -0.0, np.nan, np.inf, -np.inf, 1.0, -1.0, 0.5, 0.25, 1e-30], np.float32)
+    P = rng.choice(vals, n).astype(np.float32)
+    for K in (1, n // 3, n - 2):
+        assert np.array_equal(gpu_mask(P, K, cuda), O.topk_mask(P, K)), (n, K)
+
+
 def test_large_input_many_ctas(cuda):
     rng = np.random.default_rng(11)
     n = 8 * 1024 * 1024 + 12345
