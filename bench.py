@@ -561,6 +561,25 @@ def cpu_oracle_step(wl, env, layers, dev):
     return total / layers * wl.L, rows
 
 
+def cpu_oracle_compaction(wl, env, layer=0):
+    """CPU oracle (single thread) prune-and-pack of one layer of the dense caches,
+    the same bytes the GPU pack moves; returns seconds per full pass (scaled by L)
+    and the layer's kept rows."""
+    import oracle as O
+    import paper_2609_32663_gb300.dkv as dkv
+    ln, off, ioff, idx = dkv.dkv_plan_read(env["plan"])
+    NHl = wl.B * wl.Hkv
+    a, b = layer * NHl, (layer + 1) * NHl
+    m = O.Mapping(ln[a:b].copy(), (off[a:b + 1] - off[a]).copy(), (ioff[a:b + 1] - ioff[a]).copy(),
+                  idx[int(ioff[a]):int(ioff[b])].copy())
+    Kh = I.bf16_bits(env["K"][layer])
+    Vh = I.bf16_bits(env["V"][layer])
+    t0 = time.perf_counter()
+    O.compact(m, 1, wl.B, wl.Hkv, Kh, Vh, env["T_stride"])
+    t = time.perf_counter() - t0
+    return t * wl.L, int(ln[a:b].sum())
+
+
 def cpu_model():
     try:
         with open("/proc/cpuinfo") as f:
@@ -695,6 +714,12 @@ def run_dkv(args, dist):
                                "sample": f"fp64 scalar oracle, {layers} of {wl.L} layers of one decode step "
                                          f"({rows} rows x G={wl.G} heads), scaled x{wl.L / layers:g} to a step",
                                "cpu": cpu_model(), "nproc": os.cpu_count()}
+        with nvtx("CPU oracle compaction"):
+            t_cc, kept_cc = cpu_oracle_compaction(wl, env)
+        res["cpu_compaction"] = {"ms_per_pass": round(t_cc * 1e3, 1), "cores": 1, "kind": "oracle",
+                                 "gbs": round(2 * 512 * kept_cc * wl.L / t_cc / 1e9, 2),
+                                 "sample": f"row-by-row pack of layer 0 of {wl.L} ({kept_cc} kept rows), "
+                                           f"scaled x{wl.L} to a pass"}
     if not args.profile:
         with nvtx("pattern export"):
             res["pattern_export"] = time_topk(wl, dev)
