@@ -561,6 +561,30 @@ def cpu_oracle_step(wl, env, layers, dev):
     return total / layers * wl.L, rows
 
 
+def cpu_oracle_step_threads(wl, env, threads):
+    """The CPU oracle on `threads` layers of one decode step at once, one layer a
+    thread (the oracle's C call releases the interpreter lock); returns seconds
+    per full step (wall time scaled by L / threads) and the threads used."""
+    import concurrent.futures as cf
+
+    import oracle as O
+    import paper_2609_32663_gb300.dkv as dkv
+    ln, off, ioff, idx = dkv.dkv_plan_read(env["plan"])
+    NHl = wl.B * wl.Hkv
+    q, _, _ = I.decode_inputs(wl, 1, seed_offset=3)
+    n = max(1, min(threads, wl.L))
+    jobs = []
+    for layer in range(n):
+        lo, hi = int(off[layer * NHl]), int(off[(layer + 1) * NHl])
+        jobs.append((layer, O.Mapping(ln, off - lo, ioff, idx), I.bf16_bits(q[0, layer]),
+                     I.bf16_bits(env["Kc"][lo:hi]), I.bf16_bits(env["Vc"][lo:hi])))
+    with cf.ThreadPoolExecutor(max_workers=n) as ex:
+        t0 = time.perf_counter()
+        list(ex.map(lambda j: O.decode(j[1], j[0], wl.B, wl.H, wl.Hkv, j[2], j[3], j[4]), jobs))
+        t = time.perf_counter() - t0
+    return t * wl.L / n, n
+
+
 def cpu_oracle_compaction(wl, env, layer=0):
     """CPU oracle (single thread) prune-and-pack of one layer of the dense caches,
     the same bytes the GPU pack moves; returns seconds per full pass (scaled by L)
@@ -714,6 +738,12 @@ def run_dkv(args, dist):
                                "sample": f"fp64 scalar oracle, {layers} of {wl.L} layers of one decode step "
                                          f"({rows} rows x G={wl.G} heads), scaled x{wl.L / layers:g} to a step",
                                "cpu": cpu_model(), "nproc": os.cpu_count()}
+        with nvtx("CPU oracle, all cores"):
+            t_all, n_thr = cpu_oracle_step_threads(wl, env, os.cpu_count() or 1)
+        res["cpu_baseline_all_cores"] = {"value": round(t_all * 1e6, 1), "unit": UNIT, "cores": n_thr,
+                                         "kind": "oracle",
+                                         "sample": f"{n_thr} layers of one decode step, one a thread, "
+                                                   f"scaled x{wl.L / n_thr:g} to a step"}
         with nvtx("CPU oracle compaction"):
             t_cc, kept_cc = cpu_oracle_compaction(wl, env)
         res["cpu_compaction"] = {"ms_per_pass": round(t_cc * 1e3, 1), "cores": 1, "kind": "oracle",
