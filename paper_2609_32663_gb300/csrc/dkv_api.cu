@@ -32,7 +32,8 @@ struct dkv_plan {
     float* d_work = nullptr;    // split-K partials
     int32_t* d_slab_count = nullptr;  // [B*H_kv][G] arrival counters of the fused combine
     dkv::DecodeConfig cfg{};        // the decode step's kernel
-    dkv::DecodeConfig cfg_multi{};  // the multi-query kernel (tensor-core plans)
+    dkv::DecodeConfig cfg_multi1{};  // multi-query, one column tile (tensor-core plans)
+    dkv::DecodeConfig cfg_multi{};   // multi-query, two column tiles (tensor-core plans)
     int64_t slots = 0;              // (CTA, slab) partial slots: CTAs + slabs of a layer
     int nctas_cap = 0, warps_cap = 0, cols_cap = 0;  // workspace sized for these
     int use_mma = 0;  // tensor-core decode kernel (needs the cache's row count for its tensor maps)
@@ -136,11 +137,12 @@ dkv_status finish_plan(dkv_plan* p)
     p->use_mma = p->total_rows >= 1 && p->total_rows <= dkv::kMaxMmaRows;
     cudaError_t e;
     if (p->use_mma) {
-        if ((e = dkv::decode_config_mma(p->G, p->B, 1, &p->cfg)) != cudaSuccess) return cuda_fail(e, "decode_config");
-        if ((e = dkv::decode_config_mma(p->G, p->B, 2, &p->cfg_multi)) != cudaSuccess)
+        if ((e = dkv::decode_config_mma(p->G, p->B, 0, &p->cfg)) != cudaSuccess) return cuda_fail(e, "decode_config");
+        if ((e = dkv::decode_config_mma(p->G, p->B, 1, &p->cfg_multi1)) != cudaSuccess ||
+            (e = dkv::decode_config_mma(p->G, p->B, 2, &p->cfg_multi)) != cudaSuccess)
             return cuda_fail(e, "decode_config (multi-query)");
-        p->nctas_cap = std::max(p->cfg.nctas, p->cfg_multi.nctas);
-        p->warps_cap = std::max(p->cfg.nwarps, p->cfg_multi.nwarps);
+        p->nctas_cap = std::max({p->cfg.nctas, p->cfg_multi1.nctas, p->cfg_multi.nctas});
+        p->warps_cap = std::max({p->cfg.nwarps, p->cfg_multi1.nwarps, p->cfg_multi.nwarps});
         p->cols_cap = dkv::kMaxCols;
     } else {
         if ((e = dkv::decode_config(p->G, p->B, &p->cfg)) != cudaSuccess) return cuda_fail(e, "decode_config");
@@ -622,7 +624,8 @@ dkv_status dkv_decode_multi(const dkv_plan* p, int32_t layer, const void* q, int
         return fail(DKV_ERR_INVALID_ARG, "multi-query decode needs the tensor-core kernel (a cache of < 2^31 rows)");
     a.Q = num_queries;
     a.NC = num_queries * p->G;
-    const dkv::DecodeConfig& cfg = a.NC > 8 ? p->cfg_multi : p->cfg;
+    // Q = 1 runs the decode step's kernel; more queries the multi-query kernels.
+    const dkv::DecodeConfig& cfg = num_queries == 1 ? p->cfg : (a.NC > 8 ? p->cfg_multi : p->cfg_multi1);
     a.nctas = cfg.nctas;
     dkv::CacheMaps maps;
     const cudaError_t e = dkv::make_cache_maps(a.Kc, a.Vc, p->total_rows, &maps);

@@ -53,23 +53,31 @@ struct MK {
 // Stages per warp, warps per CTA. One column tile (the decode step): more warps
 // hide more of a tile's latency chain (8 dependent score MMAs, softmax, 16
 // output MMAs), and at the end of a pass the CTA's (slab, column) merge tasks
-// spread over more warps, which counts for G > 4 (G tasks per slab). Two column
-// tiles (multi-query): twice the accumulators still fit 12 warps without
-// spills, and two stages hold a 16-column final state; measured against 8
-// warps x 3 stages, 2 % faster at G = 7 and 0.3 % at G = 4.
+// spread over more warps, which counts for G > 4 (G tasks per slab). Multi-query
+// with one column tile: Q G columns give up to 8 merge tasks per slab, so 16
+// warps x 1 stage (measured against 12 x 2: 7-10 % faster at Q = 2). Two column
+// tiles: twice the accumulators still fit 12 warps without spills, and two
+// stages hold a 16-column final state; measured against 8 warps x 3 stages,
+// 2 % faster at G = 7 and 0.3 % at G = 4.
 #ifndef DKV_MMA_CFG_SMALL_G
 #define DKV_MMA_CFG_SMALL_G 2, 12
 #endif
 #ifndef DKV_MMA_CFG_LARGE_G
 #define DKV_MMA_CFG_LARGE_G 1, 16
 #endif
+#ifndef DKV_MMA_CFG_MULTI1
+#define DKV_MMA_CFG_MULTI1 1, 16
+#endif
 #ifndef DKV_MMA_CFG_MULTI
 #define DKV_MMA_CFG_MULTI 2, 12
 #endif
-template <int G, int NT>
+template <int G, int NT, bool MULTI>
 using MKFor = typename std::conditional<
     (NT > 1), MK<G, NT, DKV_MMA_CFG_MULTI>,
-    typename std::conditional<(G <= 4), MK<G, 1, DKV_MMA_CFG_SMALL_G>, MK<G, 1, DKV_MMA_CFG_LARGE_G>>::type>::type;
+    typename std::conditional<
+        MULTI, MK<G, 1, DKV_MMA_CFG_MULTI1>,
+        typename std::conditional<(G <= 4), MK<G, 1, DKV_MMA_CFG_SMALL_G>,
+                                  MK<G, 1, DKV_MMA_CFG_LARGE_G>>::type>::type>::type;
 
 // ------------------------------------------------------------ PTX wrappers
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar,
@@ -330,10 +338,10 @@ __device__ __forceinline__ void write_mma_out(const DecodeArgs& a, const MmaStat
 // MULTI: columns are Q x G with Q from the arguments (multi-query); otherwise
 // the G heads of the decode step, fixed at compile time.
 template <int G, int NT, bool FUSED, bool MULTI>
-__global__ void __launch_bounds__(MKFor<G, NT>::NW * 32, 1)
+__global__ void __launch_bounds__(MKFor<G, NT, MULTI>::NW * 32, 1)
     decode_mma_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ CacheMaps maps)
 {
-    using C = MKFor<G, NT>;
+    using C = MKFor<G, NT, MULTI>;
     constexpr int NCC = MULTI ? 0 : G;
     const int NC = MULTI ? a.NC : G;
     constexpr int TR = C::TR, NS = C::NS, NW = C::NW;
@@ -556,33 +564,32 @@ __global__ void __launch_bounds__(MKFor<G, NT>::NW * 32, 1)
 template <int G, int NT, bool FUSED, bool MULTI>
 cudaError_t launch_mma_g(const DecodeArgs& a, const CacheMaps& maps, const DecodeConfig& cfg, cudaStream_t st)
 {
-    return launch_pdl(decode_mma_kernel<G, NT, FUSED, MULTI>, cfg.nctas, MKFor<G, NT>::NW * 32, cfg.smem_bytes, st, a,
-                      maps);
+    using C = MKFor<G, NT, MULTI>;
+    // The configuration must be this kernel's: its warps and shared-memory layout.
+    if (cfg.nwarps != C::NW || cfg.smem_bytes < C::bytes(a.B)) return cudaErrorInvalidConfiguration;
+    return launch_pdl(decode_mma_kernel<G, NT, FUSED, MULTI>, cfg.nctas, C::NW * 32, cfg.smem_bytes, st, a, maps);
 }
 
-// Launch configuration of the tensor-core kernel with NT column tiles (the
-// multi-query kernel, NT = 2, exists fused only).
-template <int G, int NT>
+// Launch configuration of the tensor-core kernels of one kind: the decode step
+// (NT = 1, partial and fused), or multi-query with NT column tiles (fused only).
+template <int G, int NT, bool MULTI>
 cudaError_t config_mma_g(int B, DecodeConfig* cfg)
 {
-    using C = MKFor<G, NT>;
+    using C = MKFor<G, NT, MULTI>;
     const int smem = C::bytes(B);
     cudaError_t e;
-    if constexpr (NT == 1) {
+    if constexpr (!MULTI) {
         if ((e = cudaFuncSetAttribute(decode_mma_kernel<G, NT, false, false>,
                                       cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess)
             return e;
-        if ((e = cudaFuncSetAttribute(decode_mma_kernel<G, NT, true, false>,
-                                      cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess)
-            return e;
     }
-    if ((e = cudaFuncSetAttribute(decode_mma_kernel<G, NT, true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if ((e = cudaFuncSetAttribute(decode_mma_kernel<G, NT, true, MULTI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   smem)) != cudaSuccess)
         return e;
     int dev = 0, sms = 0, per_sm = 0;
     if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
     if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-    if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_mma_kernel<G, NT, true, true>, C::NW * 32,
+    if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_mma_kernel<G, NT, true, MULTI>, C::NW * 32,
                                                            smem)) != cudaSuccess)
         return e;
     if (per_sm < 1) return cudaErrorInvalidConfiguration;
@@ -628,11 +635,13 @@ cudaError_t make_cache_maps(const void* Kc, const void* Vc, int64_t rows, CacheM
     return cudaSuccess;
 }
 
-cudaError_t decode_config_mma(int G, int B, int NT, DecodeConfig* cfg)
+cudaError_t decode_config_mma(int G, int B, int kind, DecodeConfig* cfg)
 {
-    if (B < 1 || B > kMaxB || NT < 1 || NT > 2) return cudaErrorInvalidValue;
-#define DKV_CFG_CASE(g) \
-    case g: return NT == 1 ? config_mma_g<g, 1>(B, cfg) : config_mma_g<g, 2>(B, cfg);
+    if (B < 1 || B > kMaxB || kind < 0 || kind > 2) return cudaErrorInvalidValue;
+#define DKV_CFG_CASE(g)                                                               \
+    case g:                                                                           \
+        return kind == 0 ? config_mma_g<g, 1, false>(B, cfg)                          \
+                         : (kind == 1 ? config_mma_g<g, 1, true>(B, cfg) : config_mma_g<g, 2, true>(B, cfg));
     switch (G) {
         DKV_CFG_CASE(1)
         DKV_CFG_CASE(2)

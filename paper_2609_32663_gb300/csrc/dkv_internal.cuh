@@ -120,9 +120,10 @@ struct CacheMaps {
 };
 constexpr int64_t kMaxMmaRows = ((int64_t)1 << 31) - 16;
 cudaError_t make_cache_maps(const void* Kc, const void* Vc, int64_t rows, CacheMaps* maps);
-// Launch configuration of the tensor-core kernel with NT tiles of 8 columns:
-// NT = 1 for up to 8 columns (the decode step), 2 for up to 16 (multi-query).
-cudaError_t decode_config_mma(int G, int B, int NT, DecodeConfig* cfg);
+// Launch configuration of the tensor-core kernels of one kind: 0 = the decode
+// step (G columns), 1 = multi-query with one tile of 8 columns, 2 = multi-query
+// with two tiles (up to 16 columns).
+cudaError_t decode_config_mma(int G, int B, int kind, DecodeConfig* cfg);
 cudaError_t launch_decode_mma_partial(const DecodeArgs& a, const CacheMaps& maps, const DecodeConfig& cfg,
                                       cudaStream_t st);
 cudaError_t launch_decode_mma_fused(const DecodeArgs& a, const CacheMaps& maps, const DecodeConfig& cfg,
