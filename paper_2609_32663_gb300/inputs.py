@@ -63,6 +63,11 @@ WORKLOADS = {
                                   W=_w(4096, 32), pattern="bernoulli", rate=0.35, seed=1),
     "llama8b-32k": Workload("llama8b-32k", L=32, H=32, Hkv=8, T=32768, B=1, D=64,
                             W=_w(32768, 64), pattern="profile", rate=0.35, seed=2),
+    # All 256 slabs of the model at a 16K context: about 5 GB on the device with
+    # the page-backed copies of the in-place path, a small case for profiles of
+    # the kernels whose parallelism is one CTA per slab.
+    "llama8b-16k": Workload("llama8b-16k", L=32, H=32, Hkv=8, T=16384, B=1, D=32,
+                            W=_w(16384, 32), pattern="profile", rate=0.35, seed=6),
     "llama8b-128k": Workload("llama8b-128k", L=32, H=32, Hkv=8, T=131072, B=1, D=128,
                              W=_w(131072, 128), pattern="profile", rate=0.346,
                              physical_target=0.346, outlier_frac=0.01, seed=3),
