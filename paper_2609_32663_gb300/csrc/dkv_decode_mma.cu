@@ -565,9 +565,11 @@ template <int G, int NT, bool FUSED, bool MULTI>
 cudaError_t launch_mma_g(const DecodeArgs& a, const CacheMaps& maps, const DecodeConfig& cfg, cudaStream_t st)
 {
     using C = MKFor<G, NT, MULTI>;
-    // The configuration must be this kernel's: its warps and shared-memory layout.
-    if (cfg.nwarps != C::NW || cfg.smem_bytes < C::bytes(a.B)) return cudaErrorInvalidConfiguration;
-    return launch_pdl(decode_mma_kernel<G, NT, FUSED, MULTI>, cfg.nctas, C::NW * 32, cfg.smem_bytes, st, a, maps);
+    // The configuration must be this kernel's: its warps and shared-memory layout;
+    // the grid is the call's CTA count (at most the configuration's).
+    if (cfg.nwarps != C::NW || cfg.smem_bytes < C::bytes(a.B) || a.nctas < 1 || a.nctas > cfg.nctas)
+        return cudaErrorInvalidConfiguration;
+    return launch_pdl(decode_mma_kernel<G, NT, FUSED, MULTI>, a.nctas, C::NW * 32, cfg.smem_bytes, st, a, maps);
 }
 
 // Launch configuration of the tensor-core kernels of one kind: the decode step
