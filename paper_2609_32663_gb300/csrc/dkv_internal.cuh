@@ -84,9 +84,9 @@ struct DecodeArgs {
 constexpr int kMaxCols = 16;
 
 struct DecodeConfig {
-    int nctas;        // grid of the partial kernel
-    int nwarps;       // warps per CTA of the partial kernel
-    int smem_bytes;   // dynamic shared memory of the partial kernel
+    int nctas;        // the kernel's full grid (one CTA per SM); a call may use fewer (DecodeArgs::nctas)
+    int nwarps;       // warps per CTA of the kernel
+    int smem_bytes;   // dynamic shared memory of the kernel
 };
 
 // Floats of split-K workspace a decode call needs for group size G: one
