@@ -62,7 +62,10 @@ dkv_status ok()
 }
 
 // Host-side fault injection for tests: DKV_FAULT=alloc makes the next device
-// allocations fail, DKV_FAULT=launch makes kernel launches report failure.
+// allocations fail, DKV_FAULT=launch makes kernel launches report failure, and
+// DKV_FAULT=copy gives the tensor-core decode tensor maps whose boxes deliver
+// half the bytes a stage expects, so every bounded copy wait runs out (the
+// kernel then sets DKV_DEV_TMA_TIMEOUT and returns; nothing faults).
 bool fault(const char* what)
 {
     const char* f = std::getenv("DKV_FAULT");
@@ -606,7 +609,7 @@ dkv_status launch_split_k(const dkv_plan* p, const dkv::DecodeArgs& a, bool fuse
     const char* what = fused ? "decode kernel" : "decode partial kernel";
     if (p->use_mma) {
         dkv::CacheMaps maps;
-        const cudaError_t e = dkv::make_cache_maps(a.Kc, a.Vc, p->total_rows, &maps);
+        const cudaError_t e = dkv::make_cache_maps(a.Kc, a.Vc, p->total_rows, &maps, fault("copy"));
         if (e != cudaSuccess) return cuda_fail(e, "tensor maps of the packed caches");
         return launched(fused ? dkv::launch_decode_mma_fused(a, maps, p->cfg, stream)
                               : dkv::launch_decode_mma_partial(a, maps, p->cfg, stream),
@@ -648,7 +651,7 @@ dkv_status dkv_decode_multi(const dkv_plan* p, int32_t layer, const void* q, int
     const dkv::DecodeConfig& cfg = num_queries == 1 ? p->cfg : (a.NC > 8 ? p->cfg_multi : p->cfg_multi1);
     a.nctas = launch_ctas(p, layer, cfg);
     dkv::CacheMaps maps;
-    const cudaError_t e = dkv::make_cache_maps(a.Kc, a.Vc, p->total_rows, &maps);
+    const cudaError_t e = dkv::make_cache_maps(a.Kc, a.Vc, p->total_rows, &maps, fault("copy"));
     if (e != cudaSuccess) return cuda_fail(e, "tensor maps of the packed caches");
     st = launched(dkv::launch_decode_mma_fused(a, maps, cfg, stream), "multi-query decode kernel");
     return st == DKV_OK ? ok() : st;

@@ -119,7 +119,7 @@ struct CacheMaps {
     CUtensorMap k, v;
 };
 constexpr int64_t kMaxMmaRows = ((int64_t)1 << 31) - 16;
-cudaError_t make_cache_maps(const void* Kc, const void* Vc, int64_t rows, CacheMaps* maps);
+cudaError_t make_cache_maps(const void* Kc, const void* Vc, int64_t rows, CacheMaps* maps, bool short_boxes = false);
 // Launch configuration of the tensor-core kernels of one kind: 0 = the decode
 // step (G columns), 1 = multi-query with one tile of 8 columns, 2 = multi-query
 // with two tiles (up to 16 columns).

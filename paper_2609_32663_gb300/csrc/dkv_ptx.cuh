@@ -9,7 +9,8 @@
 namespace dkv {
 namespace {
 
-constexpr int kWaitSpins = 1 << 22;  // bound on mbarrier polls (each poll may suspend)
+constexpr int kWaitSpins = 1 << 22;                 // bound on mbarrier polls (each poll may suspend)
+constexpr unsigned long long kWaitNs = 2000000000ull;  // and on the time a wait may take: 2 s
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p)
 {
@@ -40,11 +41,24 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
     return ok != 0;
 }
 
-// Bounded wait: false when the phase did not complete within kWaitSpins polls.
+__device__ __forceinline__ unsigned long long global_ns()
+{
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Bounded wait: false when the phase did not complete within kWaitSpins polls
+// or kWaitNs nanoseconds, whichever comes first (a poll's suspension is
+// system-defined, so the count alone does not bound the time).
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity)
 {
-    for (int i = 0; i < kWaitSpins; ++i)
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = global_ns();
+    for (int i = 1; i < kWaitSpins; ++i) {
         if (mbar_try_wait(bar, parity)) return true;
+        if ((i & 63) == 0 && global_ns() - t0 > kWaitNs) return false;
+    }
     return false;
 }
 

@@ -34,7 +34,7 @@ constexpr int kTkThreads = 512;
 constexpr int kTkWarps = kTkThreads / 32;
 constexpr int kTkMaxCtas = 2048;
 constexpr int kTkMinPerCta = 2048;        // entries per CTA before the grid grows
-constexpr int kTkSpins = 1 << 24;         // bound on barrier polls (each an L2 round trip)
+constexpr int kTkSpins = 1 << 24;         // bound on barrier polls (each an L2 round trip), and 2 s
 constexpr int kTkSmem = kTkWarps * 1024 * 4;  // per-warp histograms of the last digit
 
 // Workspace (uint32): status, barrier counter, histograms of the three digit
@@ -75,10 +75,17 @@ __device__ bool grid_barrier(uint32_t* ws, uint32_t phase, int* ok_sh)
         asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(ctr) : "memory");
         const uint32_t target = phase * gridDim.x;
         int ok = 0;
+        unsigned long long t0;
+        asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t0));
         for (int i = 0; i < kTkSpins; ++i) {
             if (ld_acquire(ctr) >= target) {
                 ok = 1;
                 break;
+            }
+            if ((i & 255) == 255) {  // and at most 2 s
+                unsigned long long t;
+                asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+                if (t - t0 > 2000000000ull) break;
             }
         }
         if (!ok) atomicOr(ws + kWsStatus, 1u);

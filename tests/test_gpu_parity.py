@@ -279,6 +279,29 @@ def test_injected_launch_failure(monkeypatch):
     c.close()
 
 
+def test_copy_wait_runs_out_and_reports(monkeypatch):
+    """DKV_FAULT=copy gives the decode kernel tensor maps whose boxes bring half
+    the bytes each stage's mbarrier expects: every copy wait runs out at its
+    bound (2 s or 2^22 polls), the kernel sets DKV_DEV_TMA_TIMEOUT, drains and
+    returns. Nothing faults; the context stays usable and the next call is
+    exact again."""
+    import time
+    w = wl(H=8, Hkv=2, T=6000, D=8, W=606, seed=23)
+    c = Case(w)
+    q = torch.zeros((w.B, w.H, 128), dtype=torch.bfloat16, device=c.dev)
+    out = torch.empty((w.B, w.H, 128), dtype=torch.float32, device=c.dev)
+    monkeypatch.setenv("DKV_FAULT", "copy")
+    t0 = time.time()
+    dkv.dkv_decode_attn(c.plan, 0, q, None, None, None, c.Kc, c.Vc, out)
+    torch.cuda.synchronize()
+    elapsed = time.time() - t0
+    monkeypatch.delenv("DKV_FAULT")
+    assert dkv.dkv_plan_status(c.plan, clear=True) & dkv.DKV_DEV_TMA_TIMEOUT
+    assert elapsed < 60
+    c.decode_steps(1, append=False)  # exact again; checks the status word is clear
+    c.close()
+
+
 def test_unaligned_pointer_rejected():
     w = wl(H=4, Hkv=1, T=2000, D=2, W=600)
     c = Case(w)
