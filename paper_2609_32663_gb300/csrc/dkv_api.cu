@@ -65,7 +65,9 @@ dkv_status ok()
 // allocations fail, DKV_FAULT=launch makes kernel launches report failure, and
 // DKV_FAULT=copy gives the tensor-core decode tensor maps whose boxes deliver
 // half the bytes a stage expects, so every bounded copy wait runs out (the
-// kernel then sets DKV_DEV_TMA_TIMEOUT and returns; nothing faults).
+// kernel then sets DKV_DEV_TMA_TIMEOUT and returns; nothing faults), and
+// DKV_FAULT=barrier makes the Top-K export's grid barriers wait for a CTA that
+// does not exist (the first wait runs out and sets the workspace status word).
 bool fault(const char* what)
 {
     const char* f = std::getenv("DKV_FAULT");
@@ -700,7 +702,7 @@ dkv_status dkv_topk_mask(const float* P, int64_t n, int64_t K, uint8_t* M, void*
             return fail(DKV_ERR_INVALID_ARG, "workspace: need %lld bytes, 4-byte aligned",
                         (long long)dkv::topk_workspace_bytes());
     }
-    const dkv_status st = launched(dkv::launch_topk(P, n, K, M, workspace, stream), "top-k kernels");
+    const dkv_status st = launched(dkv::launch_topk(P, n, K, M, workspace, stream, fault("barrier")), "top-k kernels");
     return st == DKV_OK ? ok() : st;
 }
 

@@ -138,6 +138,9 @@ int64_t topk_workspace_bytes();
 // the release of the others (synchronises the device first).
 void vmm_pages_to_keep(const int32_t* len, int64_t nslabs, int64_t T_stride, int64_t reserve, int64_t guard,
                        int64_t row_bytes, int64_t page, int64_t npages, uint8_t* keep);
-cudaError_t launch_topk(const float* P, int64_t n, int64_t K, uint8_t* M, void* workspace, cudaStream_t st);
+// phantom_cta (fault injection): the grid barriers wait for one CTA more than
+// the grid has, so the first wait runs out at its bound.
+cudaError_t launch_topk(const float* P, int64_t n, int64_t K, uint8_t* M, void* workspace, cudaStream_t st,
+                        bool phantom_cta = false);
 
 }  // namespace dkv

@@ -66,14 +66,14 @@ __device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p)
 // Grid barrier number `phase` (1, 2, ...): every CTA arrives once per phase on
 // a counter zeroed before the launch. Bounded: false after kTkSpins polls (the
 // status word is then set), and the caller returns.
-__device__ bool grid_barrier(uint32_t* ws, uint32_t phase, int* ok_sh)
+__device__ bool grid_barrier(uint32_t* ws, uint32_t phase, uint32_t expected, int* ok_sh)
 {
     __syncthreads();
     if (threadIdx.x == 0) {
         uint32_t* ctr = ws + kWsBarrier;
         __threadfence();  // this CTA's histogram and count writes, ordered by the CTA barrier above
         asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(ctr) : "memory");
-        const uint32_t target = phase * gridDim.x;
+        const uint32_t target = phase * expected;
         int ok = 0;
         unsigned long long t0;
         asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t0));
@@ -199,8 +199,10 @@ __device__ void select_bin(const uint32_t* g, int nbins, uint32_t rank, uint32_t
     __syncthreads();
 }
 
+// arrivals: the CTAs each grid barrier counts, gridDim.x (one more only under
+// fault injection, so that the first barrier's wait runs out).
 __global__ void __launch_bounds__(kTkThreads) topk_kernel(const float* __restrict__ P, int n, uint32_t K,
-                                                          uint8_t* __restrict__ M, uint32_t* ws)
+                                                          uint8_t* __restrict__ M, uint32_t* ws, uint32_t arrivals)
 {
     extern __shared__ uint32_t h[];  // [kTkWarps][1024]: phase 3's per-warp histograms; [2048] before
     __shared__ uint32_t scratch[kTkWarps];
@@ -215,17 +217,17 @@ __global__ void __launch_bounds__(kTkThreads) topk_kernel(const float* __restric
 
     // 1: top 11 bits
     histogram<false>(P, wlo, whi, lane, h, 2048, 21, 2047u, 0, 0u, ws + kWsH1);
-    if (!grid_barrier(ws, 1, &ok_sh)) return;
+    if (!grid_barrier(ws, 1, arrivals, &ok_sh)) return;
     select_bin(ws + kWsH1, 2048, K, scratch, &sel_bin, &sel_rank);
     const uint32_t d1 = sel_bin, k1 = sel_rank;
     // 2: bits 20-10 of the keys in bin d1
     histogram<false>(P, wlo, whi, lane, h, 2048, 10, 2047u, 11, d1, ws + kWsH2);
-    if (!grid_barrier(ws, 2, &ok_sh)) return;
+    if (!grid_barrier(ws, 2, arrivals, &ok_sh)) return;
     select_bin(ws + kWsH2, 2048, k1, scratch, &sel_bin, &sel_rank);
     const uint32_t p22 = (d1 << 11) | sel_bin, k2 = sel_rank;
     // 3: bits 9-0 of the keys matching the 22-bit prefix, per warp
     histogram<true>(P, wlo, whi, lane, h, 1024, 0, 1023u, 22, p22, ws + kWsH3);
-    if (!grid_barrier(ws, 3, &ok_sh)) return;
+    if (!grid_barrier(ws, 3, arrivals, &ok_sh)) return;
     select_bin(ws + kWsH3, 1024, k2, scratch, &sel_bin, &sel_rank);
     const uint32_t T = (p22 << 10) | sel_bin, take = sel_rank;  // take the first `take` keys equal to T
     // 4: keys equal to T per warp range (bin d3 of the warp's histogram) and per CTA
@@ -236,7 +238,7 @@ __global__ void __launch_bounds__(kTkThreads) topk_kernel(const float* __restric
         for (int w = 0; w < kTkWarps; ++w) s += wties[w];
         ws[kWsTies + blockIdx.x] = s;
     }
-    if (!grid_barrier(ws, 4, &ok_sh)) return;
+    if (!grid_barrier(ws, 4, arrivals, &ok_sh)) return;
     // 5: mark. Ties before this warp's range: the earlier CTAs', then the
     // earlier warps' of this CTA; within the range, ballots in index order.
     if (warp == 0) {
@@ -262,7 +264,8 @@ __global__ void __launch_bounds__(kTkThreads) topk_kernel(const float* __restric
 
 int64_t topk_workspace_bytes() { return (int64_t)kWsWords * 4; }
 
-cudaError_t launch_topk(const float* P, int64_t n, int64_t K, uint8_t* M, void* workspace, cudaStream_t st)
+cudaError_t launch_topk(const float* P, int64_t n, int64_t K, uint8_t* M, void* workspace, cudaStream_t st,
+                        bool phantom_cta)
 {
     cudaError_t e;
     if (n == 0) return cudaSuccess;
@@ -300,7 +303,8 @@ cudaError_t launch_topk(const float* P, int64_t n, int64_t K, uint8_t* M, void* 
     if (grid < 1) grid = 1;
     int nn = (int)n;
     uint32_t KK = (uint32_t)K;
-    void* args[] = {(void*)&P, (void*)&nn, (void*)&KK, (void*)&M, (void*)&ws};
+    uint32_t arrivals = (uint32_t)grid + (phantom_cta ? 1u : 0u);
+    void* args[] = {(void*)&P, (void*)&nn, (void*)&KK, (void*)&M, (void*)&ws, (void*)&arrivals};
     return cudaLaunchCooperativeKernel((const void*)topk_kernel, dim3(grid), dim3(kTkThreads), args, kTkSmem, st);
 }
 

@@ -120,3 +120,24 @@ def test_exported_pattern_feeds_the_map(cuda):
     om = O.map_pattern(O.topk_mask(P, K), Tc, geo)
     assert np.array_equal(ln, om.len) and np.array_equal(idx, om.idx)
     plan.close()
+
+
+def test_grid_barrier_wait_runs_out_and_reports(monkeypatch, cuda):
+    """DKV_FAULT=barrier: the export's grid barriers wait for one CTA more than
+    the grid has. The first wait runs out at its bound (2 s), the status word
+    in the workspace is set and the kernel returns; the next call is exact."""
+    import time
+    rng = np.random.default_rng(3)
+    P = rng.random(300_000).astype(np.float32)
+    K = 1000
+    Pd = torch.from_numpy(P).to(cuda)
+    Md = torch.zeros(P.shape, dtype=torch.uint8, device=cuda)
+    ws = torch.zeros(dkv.dkv_topk_workspace_bytes() // 4 + 1, dtype=torch.int32, device=cuda)
+    monkeypatch.setenv("DKV_FAULT", "barrier")
+    t0 = time.time()
+    dkv.dkv_topk_mask(Pd, K, Md, ws)
+    torch.cuda.synchronize()
+    elapsed = time.time() - t0
+    monkeypatch.delenv("DKV_FAULT")
+    assert int(ws[0].item()) != 0 and elapsed < 60
+    assert np.array_equal(gpu_mask(P, K, cuda), O.topk_mask(P, K))
