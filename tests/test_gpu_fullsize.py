@@ -64,7 +64,7 @@ def _dense_rows(wl, om, slabs, T_stride):
     return np.concatenate(out)
 
 
-@pytest.mark.parametrize("name", ["llama8b-1layer-4k", "llama8b-32k", "llama8b-128k", "llama8b-b16-ragged",
+@pytest.mark.parametrize("name", ["llama8b-1layer-4k", "llama8b-16k", "llama8b-32k", "llama8b-128k", "llama8b-b16-ragged",
                                   "qwen7b-64k-b4-r20", "qwen7b-64k-b4-r35", "qwen7b-64k-b4-r50",
                                   "llama8b-128k-head-only", "llama8b-128k-distance-only",
                                   "llama8b-128k-distance-shuffled", "llama8b-128k-fully-shuffled"])
