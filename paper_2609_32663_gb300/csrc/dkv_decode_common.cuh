@@ -308,12 +308,12 @@ __device__ void cta_tail(const DecodeArgs& a, const unsigned char* ring, int war
     static_assert(2 * NW <= 32, "one entry per lane");
     const int h_e = (lane < 2 * NW) ? ((lane & 1) ? seg_last[lane >> 1] : seg_first[lane >> 1]) : -1;
     const int p0_e = h_e >= 0 ? seg_p0[lane] : 0, p1_e = h_e >= 0 ? seg_p1[lane] : 0;
-    int prev = -1;  // slab of the nearest valid entry before this one
-#pragma unroll
-    for (int f = 0; f < 2 * NW; ++f) {
-        const int hf = __shfl_sync(kFull, h_e, f);
-        if (f < lane && hf >= 0) prev = hf;
-    }
+    // Slab of the nearest valid entry before this one (-1 if none): one ballot
+    // and one shuffle.
+    const unsigned valid = __ballot_sync(kFull, h_e >= 0);
+    const unsigned below = valid & ((1u << lane) - 1u);
+    const int hprev = __shfl_sync(kFull, h_e, below ? 31 - __clz(below) : 0);
+    const int prev = below ? hprev : -1;
     const unsigned fresh = __ballot_sync(kFull, h_e >= 0 && h_e != prev);
     const int nslab = __popc(fresh);
     const int NC = NCC ? NCC : a.NC;  // columns (query x head) per slab; NCC: known at compile time
