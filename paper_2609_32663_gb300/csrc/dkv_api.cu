@@ -30,7 +30,7 @@ struct dkv_plan {
     int32_t* d_idx = nullptr;   // [kept]
     int32_t* d_status = nullptr;
     float* d_work = nullptr;    // split-K partials
-    int32_t* d_slab_count = nullptr;  // [B*H_kv][G] arrival counters of the fused combine
+    int32_t* d_slab_count = nullptr;  // [B*H_kv][cols][2] arrival / written counters of the fused combine
     dkv::DecodeConfig cfg{};        // the decode step's kernel
     dkv::DecodeConfig cfg_multi1{};  // multi-query, one column tile (tensor-core plans)
     dkv::DecodeConfig cfg_multi{};   // multi-query, two column tiles (tensor-core plans)
@@ -65,9 +65,12 @@ dkv_status ok()
 // allocations fail, DKV_FAULT=launch makes kernel launches report failure, and
 // DKV_FAULT=copy gives the tensor-core decode tensor maps whose boxes deliver
 // half the bytes a stage expects, so every bounded copy wait runs out (the
-// kernel then sets DKV_DEV_TMA_TIMEOUT and returns; nothing faults), and
-// DKV_FAULT=barrier makes the Top-K export's grid barriers wait for a CTA that
-// does not exist (the first wait runs out and sets the workspace status word).
+// kernel then sets DKV_DEV_TMA_TIMEOUT and returns; nothing faults),
+// DKV_FAULT=merge makes the last CTA of each fused merge wait for one partial
+// more than the slab has (the wait runs out, sets DKV_DEV_MERGE_TIMEOUT and
+// skips that merge), and DKV_FAULT=barrier makes the Top-K export's grid
+// barriers wait for a CTA that does not exist (the first wait runs out and sets
+// the workspace status word).
 bool fault(const char* what)
 {
     const char* f = std::getenv("DKV_FAULT");
@@ -171,9 +174,9 @@ dkv_status finish_plan(dkv_plan* p)
     st = dalloc(&p->d_status, 1, "status word");
     if (st != DKV_OK) return st;
     if ((e = cudaMemset(p->d_status, 0, sizeof(int32_t))) != cudaSuccess) return cuda_fail(e, "cudaMemset");
-    st = dalloc(&p->d_slab_count, (size_t)p->B * p->s.H_kv * p->cols_cap, "slab counters");
+    st = dalloc(&p->d_slab_count, (size_t)2 * p->B * p->s.H_kv * p->cols_cap, "slab counters");
     if (st != DKV_OK) return st;
-    if ((e = cudaMemset(p->d_slab_count, 0, sizeof(int32_t) * p->B * p->s.H_kv * p->cols_cap)) != cudaSuccess)
+    if ((e = cudaMemset(p->d_slab_count, 0, sizeof(int32_t) * 2 * p->B * p->s.H_kv * p->cols_cap)) != cudaSuccess)
         return cuda_fail(e, "cudaMemset");
     return DKV_OK;
 }
@@ -590,6 +593,7 @@ dkv_status decode_args(const dkv_plan* p, int32_t layer, const void* q, const vo
     a->warp_ml = a->warp_o + nw * p->cols_cap * dkv::kHeadDim;
     a->out = out;
     a->slab_count = p->d_slab_count;
+    a->merge_extra = fault("merge") ? 1 : 0;
     a->status = p->d_status;
     a->B = p->B;
     a->H = p->s.H;

@@ -334,6 +334,12 @@ __device__ void cta_tail(const DecodeArgs& a, const unsigned char* ring, int war
         const unsigned same = __ballot_sync(kFull, h_e == h);
         int c0h = 0, c1h = 0;
         const int nct = FUSED ? ctas_of_slab(hp0, hp1, R, a.nctas, &c0h, &c1h) : 0;
+        // Count this CTA in for (slab, head) now, so that the atomic's round trip
+        // overlaps the merge below. Counter pair: arrivals, then partials written.
+        int32_t* ctr = FUSED ? a.slab_count + ((int64_t)h * NC + j) * 2 : nullptr;
+        int old = 0;
+        if (FUSED && nct > 1 && lane == 0)
+            asm volatile("atom.relaxed.gpu.global.add.s32 %0, [%1], 1;" : "=r"(old) : "l"(ctr) : "memory");
         float M = -INFINITY;
 #pragma unroll
         for (int f = 0; f < 2 * NW; ++f) {
@@ -369,20 +375,35 @@ __device__ void cta_tail(const DecodeArgs& a, const unsigned char* ring, int war
         reinterpret_cast<float4*>(a.work_o + (slot * NC + j) * kHeadDim)[lane] = O;
         if (lane == 0) *reinterpret_cast<float2*>(a.work_ml + (slot * NC + j) * 2) = make_float2(M, L);
         if (!FUSED) continue;
-        // Count this CTA in for (slab, head): release of the partial just written,
-        // and, for the last CTA, acquire of the others' before merging them.
         __syncwarp();
-        int last = 0;
-        if (lane == 0) {
-            int32_t* ctr = a.slab_count + (int64_t)h * NC + j;
-            int old;
-            asm volatile("atom.add.acq_rel.gpu.s32 %0, [%1], 1;" : "=r"(old) : "l"(ctr) : "memory");
-            last = (old == nct - 1) ? 1 : 0;
-            if (last) *ctr = 0;  // ready for the next call
+        if (__shfl_sync(kFull, old, 0) != nct - 1) {
+            // Not the last: release the partial just written to the last arriver.
+            if (lane == 0) asm volatile("red.release.gpu.global.add.s32 [%0], 1;" ::"l"(ctr + 1) : "memory");
+            continue;
         }
-        last = __shfl_sync(kFull, last, 0);
+        // The last arriver: acquire the other CTAs' partials once all are written
+        // (a bounded wait: every CTA that arrived is resident and writes next),
+        // make the counters ready for the next call, and merge.
+        int ok = 1;
+        if (lane == 0) {
+            ok = 0;
+            const unsigned long long t0 = global_ns();
+            for (int i = 1; i < kWaitSpins; ++i) {
+                int n;
+                asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(n) : "l"(ctr + 1) : "memory");
+                if (n == nct - 1 + a.merge_extra) {
+                    ok = 1;
+                    break;
+                }
+                if ((i & 63) == 0 && global_ns() - t0 > kWaitNs) break;
+            }
+            if (!ok) atomicOr(a.status, 0x4 /* DKV_DEV_MERGE_TIMEOUT */);
+            ctr[0] = 0;
+            ctr[1] = 0;
+        }
+        ok = __shfl_sync(kFull, ok, 0);
         __syncwarp();
-        if (last) merge_slab_head<G, 12, NCC>(a, h, j, c0h, c1h, R, lane);
+        if (ok) merge_slab_head<G, 12, NCC>(a, h, j, c0h, c1h, R, lane);
     }
 }
 

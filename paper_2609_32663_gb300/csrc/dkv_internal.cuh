@@ -68,7 +68,7 @@ struct DecodeArgs {
     float* warp_o;          // [nparts][G][128]: a warp's state for a slab it left mid-range
     float* warp_ml;         // [nparts][G][2]
     float* out;             // [B][H][128]
-    int32_t* slab_count;    // [B*Hkv][G] arrival counters of the fused merge (zero between calls)
+    int32_t* slab_count;    // [B*Hkv][cols][2] arrivals, partials written (zero between calls)
     int32_t* status;
     int B, H, Hkv, G;
     int reserve;
@@ -77,6 +77,7 @@ struct DecodeArgs {
     int nctas;              // CTAs of the split-K grid: the row partition's part count
     int Q;                  // queries per sequence (1 for the decode step); q and out are [B][Q][H][128]
     int NC;                 // columns per slab: Q * G; partial records hold NC rows of 128 + 2 floats
+    int merge_extra;        // partials a fused merge waits for beyond the other CTAs' (0; 1 injects a wait that runs out)
 };
 
 // Most columns (queries x group heads) one decode call handles; the plan's

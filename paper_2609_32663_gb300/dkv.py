@@ -21,6 +21,7 @@ LIB_PATH = os.path.join(_PKG, "libdkv.so")
 DKV_OK, DKV_ERR_INVALID_ARG, DKV_ERR_CUDA, DKV_ERR_OOM, DKV_ERR_RANGE, DKV_ERR_TIMEOUT = range(6)
 DKV_DEV_APPEND_OVERFLOW = 0x1
 DKV_DEV_TMA_TIMEOUT = 0x2
+DKV_DEV_MERGE_TIMEOUT = 0x4
 
 # Every entry point include/dkv.h declares.
 EXPORTS = ("dkv_last_error", "dkv_map_pattern", "dkv_plan_dense", "dkv_plan_query", "dkv_plan_read",

@@ -302,6 +302,30 @@ def test_copy_wait_runs_out_and_reports(monkeypatch):
     c.close()
 
 
+
+def test_merge_wait_runs_out_and_reports(monkeypatch):
+    """DKV_FAULT=merge makes the last CTA of each fused (slab, head) merge wait
+    for one CTA partial more than the slab has: the wait runs out at its bound
+    (2 s or 2^22 polls), the kernel sets DKV_DEV_MERGE_TIMEOUT, makes the slab
+    counters ready for the next call and skips that merge. Nothing faults; the
+    next call is exact again."""
+    import time
+    w = wl(H=8, Hkv=2, T=6000, D=8, W=606, seed=29)
+    c = Case(w)
+    q = torch.zeros((w.B, w.H, 128), dtype=torch.bfloat16, device=c.dev)
+    out = torch.empty((w.B, w.H, 128), dtype=torch.float32, device=c.dev)
+    monkeypatch.setenv("DKV_FAULT", "merge")
+    t0 = time.time()
+    dkv.dkv_decode_attn(c.plan, 0, q, None, None, None, c.Kc, c.Vc, out)
+    torch.cuda.synchronize()
+    elapsed = time.time() - t0
+    monkeypatch.delenv("DKV_FAULT")
+    assert dkv.dkv_plan_status(c.plan, clear=True) & dkv.DKV_DEV_MERGE_TIMEOUT
+    assert elapsed < 60
+    c.decode_steps(2, append=False)  # exact again; checks the status word is clear
+    c.close()
+
+
 def test_unaligned_pointer_rejected():
     w = wl(H=4, Hkv=1, T=2000, D=2, W=600)
     c = Case(w)
