@@ -291,9 +291,11 @@ __device__ void merge_slab_head(const DecodeArgs& a, int h, int j, int c0, int c
 // the first slab's state is in the warp record (c, w) of warp_o / warp_ml, the
 // last slab's in warp w's own ring at ring + w * warp_ring_bytes (o[G][128] then
 // (m, l)[G]). The states of each slab are merged; a slab wholly inside this CTA
-// is written out (fused), otherwise the CTA writes its partial to slot c + h
-// and, fused, counts itself in for each (slab, head): the last CTA to arrive
-// merges all CTA partials of that (slab, head).
+// is written out (fused), otherwise the CTA writes its partial to slot c + h.
+// Fused, the CTA counts itself in for each (slab, head) before merging its
+// warps' states; the last CTA to arrive waits until the others have written
+// their partials and merges them all. A CTA writes its partial right after it
+// arrives, with no wait in between, so the last arriver's wait always ends.
 template <int G, int NW, bool FUSED, int NCC>
 __device__ void cta_tail(const DecodeArgs& a, const unsigned char* ring, int warp_ring_bytes,
                          const int32_t* meta, int c, int R, int warp, int lane)
