@@ -172,3 +172,48 @@ def test_vmm_page_rule_keeps_every_needed_row(dkvmod, page):
             for b in (h * T * 256, h * T * 256 + rows * 256 - 1):
                 if rows > 0:
                     assert keep[b // page] == 1
+
+
+def test_binding_refuses_host_and_misshapen_buffers(dkvmod):
+    """The binding passes device addresses only: a host tensor, a strided view,
+    a wrong element type or a wrong size is refused with DKV_ERR_INVALID_ARG
+    before the library is called (a host address would be read by a kernel)."""
+    import torch
+    dkv = dkvmod
+    cases = [
+        (torch.zeros(8, dtype=torch.float32), {}, "CUDA tensor"),
+    ]
+    for t, kw, msg in cases:
+        with pytest.raises(dkv.DkvError) as e:
+            dkv._dev(t, "out", **kw)
+        assert e.value.status == dkv.DKV_ERR_INVALID_ARG and msg in str(e.value)
+
+    class FakeCuda:
+        """Stands in for a device tensor: the checks read only these fields."""
+        is_cuda = True
+
+        def __init__(self, dtype, n, contiguous=True):
+            self.dtype, self.n, self.c = dtype, n, contiguous
+
+        def is_contiguous(self):
+            return self.c
+
+        def numel(self):
+            return self.n
+
+        def data_ptr(self):
+            return 0x7F0000000000
+
+    f32 = (torch.float32,)
+    for t, kw, msg in [
+        (FakeCuda(torch.float32, 8, contiguous=False), {"dtypes": f32}, "contiguous"),
+        (FakeCuda(torch.float16, 8), {"dtypes": f32}, "dtype"),
+        (FakeCuda(torch.float32, 7), {"dtypes": f32, "numel": 8}, "expected 8"),
+        (FakeCuda(torch.float32, 7), {"dtypes": f32, "min_numel": 8}, "at least 8"),
+    ]:
+        with pytest.raises(dkv.DkvError) as e:
+            dkv._dev(t, "out", **kw)
+        assert e.value.status == dkv.DKV_ERR_INVALID_ARG and msg in str(e.value)
+    assert dkv._dev(FakeCuda(torch.float32, 8), "out", dtypes=f32, numel=8) == 0x7F0000000000
+    assert dkv._dev(None, "k_new") is None
+    assert dkv._dev(0x1000, "raw") == 0x1000
