@@ -217,3 +217,31 @@ def test_binding_refuses_host_and_misshapen_buffers(dkvmod):
     assert dkv._dev(FakeCuda(torch.float32, 8), "out", dtypes=f32, numel=8) == 0x7F0000000000
     assert dkv._dev(None, "k_new") is None
     assert dkv._dev(0x1000, "raw") == 0x1000
+
+
+def test_header_is_plain_c_and_links_from_c(dkvmod, tmp_path):
+    """include/dkv.h compiles as C11 (the CUDA runtime header it includes needs
+    C11), and a C program that takes the address of every declared entry point
+    links against libdkv.so and runs (no GPU call)."""
+    import shutil
+    import subprocess
+    cc = os.environ.get("CC", "gcc")
+    if shutil.which(cc) is None:
+        pytest.skip("no C compiler")
+    cuda_inc = os.path.join(os.environ.get("CUDA_HOME", "/usr/local/cuda"), "include")
+    names = declared_functions()
+    prog = tmp_path / "abi.c"
+    prog.write_text(
+        '#include <stdio.h>\n#include "dkv.h"\n'
+        "typedef void (*fn)(void);\nint main(void) {\n    const fn f[] = {\n"
+        + "".join(f"        (fn)&{n},\n" for n in names)
+        + "    };\n    int n = 0;\n"
+        "    for (unsigned i = 0; i < sizeof f / sizeof f[0]; ++i) n += f[i] != 0;\n"
+        '    printf("%d\\n", n);\n    return 0;\n}\n')
+    libdir = os.path.dirname(dkvmod.LIB_PATH)
+    exe = tmp_path / "abi"
+    subprocess.check_call([cc, "-std=c11", "-Wall", "-Wextra", "-Werror",
+                           "-I", os.path.join(ROOT, "include"), "-I", cuda_inc, str(prog), "-o", str(exe),
+                           "-L", libdir, "-ldkv", f"-Wl,-rpath,{libdir}"])
+    out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout
+    assert int(out) == len(names)
