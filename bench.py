@@ -47,7 +47,6 @@ DECODE_TRAFFIC = {
     "sha256": None,  # the kernel changed since the capture: traffic unknown until re-captured
     "dram_bytes": 194_384_896 + 3_126_272,
     "algorithmic_bytes": 376_646 * 512 + 32 * 128 * (2 + 4),
-    "capture": "profiles/decode_mma_llama8b-128k-l4.md",
 }
 
 
@@ -672,8 +671,9 @@ def run_dkv(args, dist):
     res = {
         "metric": METRIC, "value": round(t_step * 1e6, 2), "unit": UNIT, "n_gpus": dist.world,
         "steps": steps, "warmup": warmup, "ms_per_step": round(t_step * 1e3, 4),
-        "higher_is_better": False, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
-        "io_dtype": "bf16", "data": "synthetic",
+        "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16 in, fp32 accumulate; P.V with P as a bf16 hi+lo pair (~16 significant bits)",
+        "io_dtype": "bf16 q/K/V, fp32 out", "data": "synthetic",
         "config": {"workload": wl.name, "layers": wl.L, "q_heads": wl.H, "kv_heads": wl.Hkv, "head_dim": wl.head_dim,
                    "batch": wl.B, "ctx_len": [int(x) for x in env["Tc"]][:16], "bins": wl.D, "bin_width": wl.W,
                    "sink": wl.sink, "recent": wl.recent,

@@ -118,7 +118,10 @@ dkv_status dkv_plan_dense(const int32_t* ctx_len_host, int32_t B, const dkv_shap
                           int64_t T_stride, cudaStream_t stream, dkv_plan** out);
 
 /*
- * Read-only views of a plan. Any output pointer may be NULL.
+ * Read-only views of a plan. Any output pointer may be NULL. Besides the total
+ * row count and the len/off/idx views, it returns kept_rows (the size of d_idx)
+ * and d_ioff (where each slab's positions start in d_idx): a caller cannot
+ * walk d_idx without them, and dkv_decode_attn_noalloc takes d_ioff.
  * total_rows  rows the packed caches need (sum of len + reserve).
  * kept_rows   number of kept context positions (sum of len).
  * d_len       device int32 [L*B*H_kv]
@@ -313,10 +316,13 @@ dkv_status dkv_plan_status(const dkv_plan* plan, int32_t* word, int32_t clear, c
  * The split-K partials live in a fixed 8 MiB array inside the library image,
  * held on every GPU that loads the library until the process exits; a call
  * whose split-K records ((9 x SM count + B*H_kv) x G x 130 floats) do not fit gets
- * DKV_ERR_INVALID_ARG. The first call on each device looks up that array's
- * device address (a one-time set-up per device); make that first call before
- * any stream capture. Every call reuses the same array, so calls whose kernels
- * overlap on the GPU (other streams, other threads) race with each other.
+ * DKV_ERR_INVALID_ARG. The first call in a CUDA context (on each device, and
+ * again after that context is destroyed and re-created, e.g. by
+ * cudaDeviceReset) looks up the array's device address, and the first call for
+ * each (G, B) in a context sets up the kernel's launch configuration; make
+ * those first calls before any stream capture. Every call reuses the same
+ * array, so calls whose kernels overlap on the GPU (other streams, other
+ * threads) race with each other.
  * Errors: DKV_ERR_INVALID_ARG, DKV_ERR_CUDA.
  */
 dkv_status dkv_decode_attn_noalloc(const dkv_shape* s, int32_t B, int32_t layer, int32_t reserve_rows,

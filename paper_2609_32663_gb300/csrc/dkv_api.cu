@@ -35,6 +35,7 @@ struct dkv_plan {
     dkv::DecodeConfig cfg_multi1{};  // multi-query, one column tile (tensor-core plans)
     dkv::DecodeConfig cfg_multi{};   // multi-query, two column tiles (tensor-core plans)
     int64_t slots = 0;              // (CTA, slab) partial slots: CTAs + slabs of a layer
+    dkv::WorkspaceLayout work{};    // carve-up of d_work
     int nctas_cap = 0, warps_cap = 0, cols_cap = 0;  // workspace sized for these
     int use_mma = 0;  // tensor-core decode kernel (needs the cache's row count for its tensor maps)
     int64_t inplace_stride = 0;  // > 0: slab h lives at rows h * stride of the dense buffer (in place)
@@ -166,10 +167,8 @@ dkv_status finish_plan(dkv_plan* p)
         p->cols_cap = p->G;
     }
     p->slots = (int64_t)p->nctas_cap + p->B * p->s.H_kv;
-    dkv_status st = dalloc(&p->d_work,
-                           (size_t)dkv::decode_workspace_floats(p->nctas_cap, p->warps_cap, p->cols_cap,
-                                                                p->B * p->s.H_kv),
-                           "split-K workspace");
+    p->work = dkv::decode_workspace(p->nctas_cap, p->warps_cap, p->cols_cap, p->B * p->s.H_kv);
+    dkv_status st = dalloc(&p->d_work, (size_t)p->work.total, "split-K workspace");
     if (st != DKV_OK) return st;
     st = dalloc(&p->d_status, 1, "status word");
     if (st != DKV_OK) return st;
@@ -586,11 +585,12 @@ dkv_status decode_args(const dkv_plan* p, int32_t layer, const void* q, const vo
     a->len = p->d_len + (int64_t)layer * NHl;
     a->off = p->d_off + (int64_t)layer * NHl;
     a->ioff = p->d_ioff + (int64_t)layer * NHl;
-    const size_t nw = (size_t)p->nctas_cap * p->warps_cap;
-    a->work_o = p->d_work;
-    a->work_ml = a->work_o + (size_t)p->slots * p->cols_cap * dkv::kHeadDim;
-    a->warp_o = a->work_ml + (size_t)p->slots * p->cols_cap * 2;
-    a->warp_ml = a->warp_o + nw * p->cols_cap * dkv::kHeadDim;
+    a->work_o = p->d_work + p->work.work_o;
+    a->work_ml = p->d_work + p->work.work_ml;
+    a->warp_o = p->d_work + p->work.warp_o;
+    a->warp_ml = p->d_work + p->work.warp_ml;
+    if (!aligned16(a->work_o) || !aligned16(a->work_ml) || !aligned16(a->warp_o) || !aligned16(a->warp_ml))
+        return fail(DKV_ERR_INVALID_ARG, "split-K workspace regions are not 16-byte aligned");
     a->out = out;
     a->slab_count = p->d_slab_count;
     a->merge_extra = fault("merge") ? 1 : 0;

@@ -90,18 +90,35 @@ struct DecodeConfig {
     int smem_bytes;   // dynamic shared memory of the kernel
 };
 
-// Floats of split-K workspace a decode call needs for group size G: one
-// (o[128], m, l) record per head of the group for every (CTA, slab) slot
-// (nctas + slabs per layer) and for every warp of the grid.
-inline int64_t decode_workspace_floats(const DecodeConfig& c, int G, int heads_per_layer) {
-    const int64_t records = (int64_t)c.nctas + heads_per_layer + (int64_t)c.nctas * c.nwarps;
-    return records * G * (128 + 2);
+// Carve-up of the split-K workspace, in floats from its base: the (CTA, slab)
+// partials o [slots][cols][128] and (m, l) [slots][cols][2], then the warp
+// records o [warp_records][cols][128] and (m, l) [warp_records][cols][2]. Each
+// region starts on a 256-byte boundary: the kernels move o with 16-byte vector
+// accesses and (m, l) with 8-byte ones, whatever slots x cols is (an odd
+// product would otherwise leave the warp records 8-byte aligned).
+struct WorkspaceLayout {
+    int64_t work_o, work_ml, warp_o, warp_ml;  // region offsets (floats)
+    int64_t total;                             // floats of the whole workspace
+};
+constexpr int64_t kWorkAlignFloats = 64;  // 256 bytes
+inline int64_t round_up_work(int64_t n) { return (n + kWorkAlignFloats - 1) / kWorkAlignFloats * kWorkAlignFloats; }
+inline WorkspaceLayout workspace_layout(int64_t slots, int64_t warp_records, int cols)
+{
+    WorkspaceLayout w;
+    w.work_o = 0;
+    w.work_ml = w.work_o + round_up_work(slots * cols * kHeadDim);
+    w.warp_o = w.work_ml + round_up_work(slots * cols * 2);
+    w.warp_ml = w.warp_o + round_up_work(warp_records * cols * kHeadDim);
+    w.total = w.warp_ml + round_up_work(warp_records * cols * 2);
+    return w;
 }
-// The same for a workspace shared by kernels of up to `nctas` CTAs of up to
-// `nwarps` warps handling up to `cols` columns.
-inline int64_t decode_workspace_floats(int nctas, int nwarps, int cols, int heads_per_layer) {
-    const int64_t records = (int64_t)nctas + heads_per_layer + (int64_t)nctas * nwarps;
-    return records * cols * (128 + 2);
+// The workspace of kernels of up to `nctas` CTAs of up to `nwarps` warps
+// handling up to `cols` columns over a layer of `heads_per_layer` slabs: one
+// record per column for every (CTA, slab) slot (nctas + slabs) and for every
+// warp of the grid.
+inline WorkspaceLayout decode_workspace(int nctas, int nwarps, int cols, int heads_per_layer)
+{
+    return workspace_layout((int64_t)nctas + heads_per_layer, (int64_t)nctas * nwarps, cols);
 }
 // Grid and shared memory of the partial kernel for group size G on this device.
 cudaError_t decode_config(int G, int B, DecodeConfig* cfg);

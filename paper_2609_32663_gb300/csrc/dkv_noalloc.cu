@@ -16,10 +16,15 @@
 #include "dkv.h"
 #include "dkv_internal.cuh"
 
+#include <cuda.h>
+
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <map>
 #include <mutex>
+#include <tuple>
+#include <vector>
 
 namespace {
 
@@ -30,26 +35,75 @@ constexpr size_t kStatusOffset = kScratchBytes - 256;
 
 static __device__ __align__(256) unsigned char g_decode_scratch[kScratchBytes];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_setup_mu;
-void* g_scratch_addr[kMaxDevices] = {};  // device address of g_decode_scratch, per device
+// Per CUDA context (not per device ordinal: a context that is destroyed and
+// made again, e.g. after cudaDeviceReset, loads the library's module again and
+// the array moves), looked up by the context's process-unique ID:
+//   - the device address of g_decode_scratch (in host code the symbol names a
+//     host-side stand-in, never the device memory);
+//   - the fp32 decode kernel's launch configuration for each (G, B), so that a
+//     call does not set kernel attributes and query occupancy every time.
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long*);
 
-// Once per device, with that device current: the device address of the array.
-// (In host code the symbol names a host-side stand-in, never the device memory.)
-cudaError_t scratch_for_current_device(void** out)
+std::mutex g_setup_mu;
+std::vector<std::pair<unsigned long long, void*>> g_scratch_addr;  // (context ID, device address)
+std::map<std::tuple<unsigned long long, int, int>, dkv::DecodeConfig> g_configs;  // (context ID, G, B)
+
+template <class F>
+F driver_fn(const char* name)
 {
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
-    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
-    std::lock_guard<std::mutex> lk(g_setup_mu);
-    if (!g_scratch_addr[dev]) {
-        void* p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_decode_scratch);
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion(name, &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+        return nullptr;
+    return reinterpret_cast<F>(p);
+}
+
+// ID of the calling thread's current context; the runtime's primary context of
+// the current device is made current first if none is.
+cudaError_t current_context_id(unsigned long long* id)
+{
+    static const CtxGetCurrentFn get_current = driver_fn<CtxGetCurrentFn>("cuCtxGetCurrent");
+    static const CtxGetIdFn get_id = driver_fn<CtxGetIdFn>("cuCtxGetId");
+    if (!get_current || !get_id) return cudaErrorNotSupported;
+    CUcontext ctx = nullptr;
+    if (get_current(&ctx) != CUDA_SUCCESS) return cudaErrorDeviceUninitialized;
+    if (!ctx) {
+        int dev = 0;
+        cudaError_t e = cudaGetDevice(&dev);
+        if (e == cudaSuccess) e = cudaSetDevice(dev);  // initialises the device's primary context
         if (e != cudaSuccess) return e;
-        g_scratch_addr[dev] = p;
+        if (get_current(&ctx) != CUDA_SUCCESS || !ctx) return cudaErrorDeviceUninitialized;
     }
-    *out = g_scratch_addr[dev];
+    return get_id(ctx, id) == CUDA_SUCCESS ? cudaSuccess : cudaErrorDeviceUninitialized;
+}
+
+// The device address of the array and the launch configuration for (G, B) in
+// the current context, looked up on the context's first call.
+cudaError_t setup_for_current_context(int G, int B, void** scratch, dkv::DecodeConfig* cfg)
+{
+    unsigned long long id = 0;
+    cudaError_t e = current_context_id(&id);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lk(g_setup_mu);
+    void* addr = nullptr;
+    for (const auto& kv : g_scratch_addr)
+        if (kv.first == id) addr = kv.second;
+    if (!addr) {
+        e = cudaGetSymbolAddress(&addr, g_decode_scratch);
+        if (e != cudaSuccess) return e;
+        g_scratch_addr.emplace_back(id, addr);
+    }
+    const auto key = std::make_tuple(id, G, B);
+    auto it = g_configs.find(key);
+    if (it == g_configs.end()) {
+        dkv::DecodeConfig c{};
+        if ((e = dkv::decode_config(G, B, &c)) != cudaSuccess) return e;
+        it = g_configs.emplace(key, c).first;
+    }
+    *scratch = addr;
+    *cfg = it->second;
     return cudaSuccess;
 }
 
@@ -91,20 +145,18 @@ extern "C" dkv_status dkv_decode_attn_noalloc(const dkv_shape* s, int32_t B, int
         return bad(DKV_ERR_INVALID_ARG, "q/k_new/v_new/Kc/Vc/out must be 16-byte aligned");
     if (!std::isfinite(scale)) return bad(DKV_ERR_INVALID_ARG, "scale is not finite");
 
-    void* scratch = nullptr;
-    cudaError_t e = scratch_for_current_device(&scratch);
-    if (e != cudaSuccess) return bad(DKV_ERR_CUDA, "scratch set-up: %s", cudaGetErrorString(e));
     const int G = s->H / s->H_kv;
+    void* scratch = nullptr;
     dkv::DecodeConfig cfg{};
-    if ((e = dkv::decode_config(G, B, &cfg)) != cudaSuccess)
-        return bad(DKV_ERR_CUDA, "decode_config: %s", cudaGetErrorString(e));
+    cudaError_t e = setup_for_current_context(G, B, &scratch, &cfg);
+    if (e != cudaSuccess) return bad(DKV_ERR_CUDA, "scratch set-up: %s", cudaGetErrorString(e));
     const int NHl = B * s->H_kv;
-    const int64_t slots = (int64_t)cfg.nctas + NHl;
-    const size_t need = (size_t)dkv::decode_workspace_floats(cfg, G, NHl) * sizeof(float);
+    const dkv::WorkspaceLayout lay = dkv::decode_workspace(cfg.nctas, cfg.nwarps, G, NHl);
+    const size_t need = (size_t)lay.total * sizeof(float);
     if (need > kStatusOffset)
         return bad(DKV_ERR_INVALID_ARG,
                    "split-K partials need %zu bytes (%lld slots x G=%d); the static scratch holds %zu", need,
-                   (long long)slots, G, (size_t)kStatusOffset);
+                   (long long)cfg.nctas + NHl, G, (size_t)kStatusOffset);
 
     float* work = static_cast<float*>(scratch);
     int32_t* status_word = status;
@@ -124,10 +176,12 @@ extern "C" dkv_status dkv_decode_attn_noalloc(const dkv_shape* s, int32_t B, int
     a.len = d_len + (int64_t)layer * NHl;
     a.off = d_off + (int64_t)layer * NHl;
     a.ioff = d_ioff + (int64_t)layer * NHl;
-    a.work_o = work;
-    a.work_ml = a.work_o + (size_t)slots * G * dkv::kHeadDim;
-    a.warp_o = a.work_ml + (size_t)slots * G * 2;
-    a.warp_ml = a.warp_o + (size_t)cfg.nctas * cfg.nwarps * G * dkv::kHeadDim;
+    a.work_o = work + lay.work_o;
+    a.work_ml = work + lay.work_ml;
+    a.warp_o = work + lay.warp_o;
+    a.warp_ml = work + lay.warp_ml;
+    if (!aligned16(a.work_o) || !aligned16(a.work_ml) || !aligned16(a.warp_o) || !aligned16(a.warp_ml))
+        return bad(DKV_ERR_INVALID_ARG, "split-K workspace regions are not 16-byte aligned");
     a.out = out;
     a.status = status_word;
     a.B = B;

@@ -1,9 +1,14 @@
 """Seeded synthetic inputs for the Distance-KV decode path.
 
 This module only draws inputs: retention patterns M, context lengths, and the
-bf16 K/V/q tensors. It holds none of the method's arithmetic (no distance bins,
-no retention mask, no packing, no attention), so both the CUDA path and the CPU
-oracle can be fed from it without sharing any of the computation.
+bf16 K/V/q tensors. It holds none of the path's arithmetic (no distance bins, no
+retention mask, no union of positions, no packing, no attention), so both the
+CUDA path and the CPU oracle can be fed from it without sharing any of the
+computation. To hit exact budgets the pattern generators pick the top-scoring
+entries and count group columns; those helpers (the `_gen_` functions) are
+private to the generators, and no test, smoke check or benchmark takes an
+expected value from them: expected masks, maps, bytes and outputs all come from
+the oracle.
 
 The workloads stand in for the paper's efficiency setting (Sec. 4.3, App. C:
 Llama-3.1-8B and Qwen2.5-7B caches up to 128K context on one GPU). No model
@@ -105,9 +110,11 @@ def context_lengths(wl: Workload) -> np.ndarray:
     return rng.integers(lo, hi + 1, size=wl.B, dtype=np.int64).astype(np.int32)
 
 
-def topk_mask(scores: np.ndarray, k: int) -> np.ndarray:
-    """Global Top-K of a score tensor (Eq. 3 / App. A.3 shape): the k largest
-    entries become 1. Ties go to the lower flat index (stable order)."""
+def _gen_top_entries(scores: np.ndarray, k: int) -> np.ndarray:
+    """Generator-only: the k highest-scoring entries of a score tensor become 1
+    (ties to the lower flat index), which gives the profile generator an exact
+    budget of union bins. No test takes an expected mask from it: the export's
+    expected masks come from the oracle."""
     flat = scores.reshape(-1)
     k = int(max(0, min(k, flat.size)))
     order = np.argsort(-flat, kind="stable")
@@ -116,8 +123,8 @@ def topk_mask(scores: np.ndarray, k: int) -> np.ndarray:
     return out.reshape(scores.shape)
 
 
-def round_half_up(x: float) -> int:
-    """round() of App. A.3 read as floor(x + 0.5)."""
+def _gen_round(x: float) -> int:
+    """Generator-only: floor(x + 0.5), the rounding of the generators' budgets."""
     return int(np.floor(x + 0.5))
 
 
@@ -135,8 +142,8 @@ def union_bins_target(wl: Workload) -> int:
         # Overall physical retention r of a T-token context: kept rows per head
         # = S + R + K_U * W / (L * Hkv) = r * T.
         per_head_bins = (wl.physical_target * wl.T - wl.sink - wl.recent) / wl.W
-        return round_half_up(per_head_bins * wl.L * wl.Hkv)
-    return round_half_up(wl.rate * wl.L * wl.Hkv * wl.D)
+        return _gen_round(per_head_bins * wl.L * wl.Hkv)
+    return _gen_round(wl.rate * wl.L * wl.Hkv * wl.D)
 
 
 def profile_pattern(wl: Workload, rng: np.random.Generator) -> np.ndarray:
@@ -153,7 +160,7 @@ def profile_pattern(wl: Workload, rng: np.random.Generator) -> np.ndarray:
     w = rng.beta(2.0, 2.0, size=(L, Hkv, 1))
     x = (np.arange(D) / max(D - 1, 1))[None, None, :]
     score = w * (1.0 - x) + (1.0 - w) * x + 0.25 * rng.random((L, Hkv, D))
-    U = topk_mask(score, union_bins_target(wl))
+    U = _gen_top_entries(score, union_bins_target(wl))
     M = np.zeros((L, Hkv, G, D), np.uint8)
     sel = np.argwhere(U == 1)
     for (l, g, d) in sel:
@@ -187,7 +194,9 @@ def retention_probs(wl: Workload, levels: int | None = None, seed_offset: int = 
 # count below only sizes these inputs: it counts (layer, KV head, bin) columns
 # with any query head on, i.e. physical bins at full context coverage.
 
-def _union_count(M: np.ndarray, G: int) -> int:
+def _gen_group_columns(M: np.ndarray, G: int) -> int:
+    """Generator-only: (layer, KV head, bin) columns with any query head on,
+    which sizes the ablation patterns."""
     L, H, D = M.shape
     return int(M.reshape(L, H // G, G, D).max(axis=2).sum())
 
@@ -224,7 +233,7 @@ def ablate_head_only(M: np.ndarray, G: int) -> np.ndarray:
     for the union count U of M."""
     L, H, D = M.shape
     score = M.reshape(L, H // G, G, D).max(axis=2).sum(axis=2).reshape(-1)  # union bins per (l, g)
-    n_groups = int(np.floor(_union_count(M, G) / D + 0.5))
+    n_groups = int(np.floor(_gen_group_columns(M, G) / D + 0.5))
     order = np.argsort(-score, kind="stable")[:n_groups]
     keep = np.zeros(L * (H // G), np.uint8)
     keep[order] = 1
@@ -239,7 +248,7 @@ def ablate_distance_only(M: np.ndarray, G: int) -> np.ndarray:
     L, H, D = M.shape
     Hkv = H // G
     score = M.sum(axis=1).reshape(-1)  # query heads on per (l, d)
-    n_keep = int(np.floor(_union_count(M, G) / Hkv + 0.5))
+    n_keep = int(np.floor(_gen_group_columns(M, G) / Hkv + 0.5))
     order = np.argsort(-score, kind="stable")[:n_keep]
     keep = np.zeros(L * D, np.uint8)
     keep[order] = 1
@@ -330,5 +339,5 @@ def bf16_bits(t) -> np.ndarray:
 __all__ = ["Workload", "WORKLOADS", "SINK", "RECENT", "context_lengths", "make_pattern", "retention_probs",
            "ABLATIONS", "ablate_distance_shuffled", "ablate_fully_shuffled", "ablate_head_only",
            "ablate_distance_only",
-           "topk_mask", "round_half_up", "union_bins_target", "dense_kv", "decode_inputs",
+           "union_bins_target", "dense_kv", "decode_inputs",
            "bf16_bits"]

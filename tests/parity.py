@@ -1,5 +1,8 @@
 """Shared helpers of the GPU parity tests: run the CUDA path through the C ABI and
 the CPU oracle on the same seeded inputs, and compare."""
+import json
+import os
+
 import numpy as np
 import torch
 
@@ -18,14 +21,41 @@ def shapes(wl):
     return sh, geo
 
 
+def row_errors(got, want):
+    """Per output row (the last axis: one head's 128 dims for one query): max-abs
+    error and rel-L2 error (relative to the oracle row's norm; absolute for a zero
+    row, the output of an empty slab)."""
+    got = np.asarray(got, np.float64).reshape(-1, np.shape(want)[-1] if np.ndim(want) else 1)
+    want = np.asarray(want, np.float64).reshape(got.shape)
+    diff = got - want
+    err = np.abs(diff).max(axis=1) if got.size else np.zeros(0)
+    nrm = np.linalg.norm(want, axis=1)
+    dn = np.linalg.norm(diff, axis=1)
+    rel = np.where(nrm > 0, dn / np.where(nrm > 0, nrm, 1.0), dn)
+    return err, rel
+
+
 def assert_close(got, want, what=""):
+    """Every output row (each (sequence, query, head) of 128 dims) within rel-L2
+    <= REL_L2 and max-abs <= MAX_ABS of the fp64 oracle. Returns the worst row's
+    (rel-L2, max-abs); with DKV_PARITY_LOG set, also appends them to that file."""
     got = np.asarray(got, np.float64)
     want = np.asarray(want, np.float64)
+    assert got.shape == want.shape, f"{what}: shape {got.shape} != {want.shape}"
     assert np.isfinite(got).all(), f"{what}: non-finite output"
-    err = np.abs(got - want).max() if got.size else 0.0
-    nrm = np.linalg.norm(want)
-    rel = np.linalg.norm(got - want) / nrm if nrm > 0 else np.linalg.norm(got - want)
-    assert err <= MAX_ABS and rel <= REL_L2, f"{what}: max-abs {err:.3e}, rel-L2 {rel:.3e}"
+    if got.size == 0:
+        return 0.0, 0.0
+    err, rel = row_errors(got, want)
+    bad = np.flatnonzero((err > MAX_ABS) | (rel > REL_L2))
+    assert bad.size == 0, (f"{what}: {bad.size} of {err.size} rows out of tolerance; row {bad[0]}: "
+                           f"max-abs {err[bad[0]]:.3e}, rel-L2 {rel[bad[0]]:.3e}")
+    worst = (float(rel.max()), float(err.max()))
+    log = os.environ.get("DKV_PARITY_LOG")
+    if log:
+        with open(log, "a") as f:
+            f.write(json.dumps({"what": what, "rows": int(err.size), "worst_rel_l2": worst[0],
+                                "worst_max_abs": worst[1]}) + "\n")
+    return worst
 
 
 def check_map(plan, om):

@@ -55,11 +55,42 @@ def test_oracle_imports_nothing_from_the_product():
 
 
 def test_shared_input_module_holds_no_method_arithmetic():
-    """inputs.py draws seeded tensors and patterns; the keep rule, the GQA union,
-    the pack and the attention live only in the oracle and the kernels."""
+    """inputs.py draws seeded tensors and patterns. The keep rule (distance bins
+    and the retention mask), the union of positions over a group, the pack and
+    the attention live only in the oracle and the kernels."""
     imports = _py_imports(os.path.join(PKG, "inputs.py"))
     assert "oracle" not in imports
     assert not imports & {"ctypes"}
     src = open(os.path.join(PKG, "inputs.py")).read()
-    for word in ("softmax", "dkv_decode", "dkv_compact", "dkv_map_pattern"):
+    for word in ("softmax", "dkv_decode", "dkv_compact", "dkv_map_pattern", "bin_width", "keep_pos"):
         assert word not in src, word
+
+
+# The generators reach exact budgets with three helpers that resemble steps of
+# the method: a stable global top-k of scores (the shape of the pattern export),
+# floor(x + 1/2) (the export's budget rounding) and a count of group columns
+# with any head on (the size of the GQA union at full coverage). They only size
+# and select generated patterns.
+GENERATOR_ONLY = ("_gen_top_entries", "_gen_round", "_gen_group_columns")
+
+
+def test_generator_only_helpers_are_private_to_the_generators():
+    import paper_2609_32663_gb300.inputs as I
+    for name in GENERATOR_ONLY:
+        assert hasattr(I, name), name
+        assert name not in I.__all__, name
+    for name in ("topk_mask", "round_half_up", "_union_count"):
+        assert not hasattr(I, name), name
+
+
+def test_no_expected_value_comes_from_the_generator_helpers():
+    """No test, smoke() or bench.py leg calls them: every expected mask, map,
+    byte and output is the oracle's (or a hand-worked fixture's)."""
+    users = _files(os.path.join(ROOT, "tests"), (".py",)) + [os.path.join(ROOT, "__graft_entry__.py"),
+                                                            os.path.join(ROOT, "bench.py")]
+    for f in users:
+        if os.path.basename(f) == "test_separation_cpu.py":
+            continue
+        src = open(f).read()
+        for name in GENERATOR_ONLY:
+            assert name not in src, (f, name)
