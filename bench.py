@@ -97,6 +97,7 @@ def parse():
     ap.add_argument("--workload", default="llama8b-128k", choices=sorted(I.WORKLOADS))
     ap.add_argument("--no-dense", action="store_true", help="skip the dense-cache baseline")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
+    ap.add_argument("--no-workloads", action="store_true", help="skip the other workloads' lines")
     ap.add_argument("--cpu-layers", type=int, default=2, help="layers of one step the CPU oracle times")
     ap.add_argument("--profile", action="store_true", help="few steps, no baselines (for ncu)")
     return ap.parse_args()
@@ -222,6 +223,7 @@ def setup(wl, dev, reserve):
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     plan = dkv.dkv_map_pattern(M, Tc, shape, reserve_rows=reserve)
+    torch.cuda.synchronize()  # the call returns before its last kernel (the index list) ends
     map_ms = (time.perf_counter() - t0) * 1e3
     info = dkv.dkv_plan_query(plan)
     Kc = torch.empty((info.total_rows, wl.head_dim), dtype=torch.bfloat16, device=dev)
@@ -464,6 +466,129 @@ class DecodeRunner:
             torch.cuda.synchronize()
             durs.extend(e0.elapsed_time(e1) * 1e-3 for e0, e1 in evs)
         return statistics.mean(durs), len(durs)
+
+
+def workload_line(name, dev, steps, warmup, dist, peak):
+    """One more workload at full size, timed like the headline one: map, pack,
+    the decode-step graph replayed `steps` times after `warmup`, and the dense
+    baseline (same kernels, uncompressed cache). Inputs larger than L2."""
+    import torch
+
+    import paper_2609_32663_gb300.dkv as dkv
+    wl = I.WORKLOADS[name]
+    reserve = reserve_rows(steps, warmup)
+    env = setup(wl, dev, reserve)
+    try:
+        dkv.dkv_compact(env["plan"], env["K"], env["V"], env["Kc"], env["Vc"], T_stride=env["T_stride"])
+        NHl = wl.B * wl.Hkv
+        kept = env["info"].kept_rows
+        runner = DecodeRunner(wl, env["plan"], env["Kc"], env["Vc"], dev)
+        runner.capture()
+        t, _ = time_graph(runner, steps, warmup, dist)
+        t = dist.max(t)
+        del runner
+        rows = kept + wl.L * NHl * (warmup + (steps - 1) / 2.0 + 1)
+        algo = step_bytes(wl, rows)
+        out = {"us_per_step": round(t * 1e6, 2), "gb_per_step": round(algo / 1e9, 4),
+               "gbs": round(algo / t / 1e9, 1), "frac_of_hbm": round(algo / t / 1e9 / peak, 4),
+               "physical_retention": round(kept / (wl.L * wl.Hkv * float(env["Tc"].sum())), 4),
+               "steps": steps, "l2": "inputs larger than L2 (%.2f GB of K/V per step)" % (rows * 512 / 1e9)}
+        dense = dkv.dkv_plan_dense(env["Tc"], env["shape"], T_stride=env["T_stride"])
+        dr = DecodeRunner(wl, dense, env["K"], env["V"], dev)
+        dr.capture()
+        td, _ = time_graph(dr, steps, warmup, dist)
+        td = dist.max(td)
+        del dr
+        dense.close()
+        drows = wl.L * wl.Hkv * float(env["Tc"].sum()) + wl.L * NHl * (warmup + (steps - 1) / 2.0 + 1)
+        out.update({"dense_us_per_step": round(td * 1e6, 2), "dense_gbs": round(step_bytes(wl, drows) / td / 1e9, 1),
+                    "speedup_of_compacted": round(td / t, 3), "ideal_speedup": round(drows / rows, 3)})
+        return out
+    finally:
+        env["plan"].close()
+        del env
+        torch.cuda.empty_cache()
+
+
+def rotated_small_workload(name, dev, steps, warmup, dist, peak, l2_multiple=4):
+    """A workload whose caches fit in L2 (the 1-layer 4K one: 14.7 MB a step),
+    measured from HBM: N copies of the packed caches (and of the dense ones for
+    the baseline), N chosen so that they span at least `l2_multiple` x L2, and a
+    graph of N decode steps, step i on copy i (each copy with its own appended-
+    row counter). Consecutive steps read different bytes, and a copy is read
+    again only after the other N - 1, far more than L2 holds, were streamed."""
+    import torch
+
+    import paper_2609_32663_gb300.dkv as dkv
+    wl = I.WORKLOADS[name]
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    reserve = reserve_rows(steps, warmup)
+    env = setup(wl, dev, reserve)
+    try:
+        dkv.dkv_compact(env["plan"], env["K"], env["V"], env["Kc"], env["Vc"], T_stride=env["T_stride"])
+        kept = env["info"].kept_rows
+        NHl = wl.B * wl.Hkv
+        q, kn, vn = I.decode_inputs(wl, 1, device=dev)
+        q, kn, vn = q[0].contiguous(), kn[0].contiguous(), vn[0].contiguous()
+        out = torch.empty((wl.L, wl.B, wl.H, wl.head_dim), dtype=torch.float32, device=dev)
+
+        def timed(plan, K, V, rows_bytes):
+            n = max(2, -(-l2_multiple * l2 // rows_bytes))
+            caches = [(K.clone(), V.clone(), torch.zeros(wl.B, dtype=torch.int32, device=dev)) for _ in range(n)]
+
+            def launch():
+                for Kx, Vx, na in caches:
+                    for layer in range(wl.L):
+                        dkv.dkv_decode_attn(plan, layer, q[layer], kn[layer], vn[layer], na, Kx, Vx, out[layer])
+                    dkv.dkv_advance(plan, na)
+
+            st = torch.cuda.Stream()
+            st.wait_stream(torch.cuda.current_stream())
+            with torch.cuda.stream(st):
+                launch()
+            torch.cuda.current_stream().wait_stream(st)
+            torch.cuda.synchronize()
+            for _, _, na in caches:
+                na.zero_()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                launch()
+            reps = max(1, -(-steps // n))
+            for _ in range(max(1, -(-warmup // n))):
+                g.replay()
+            torch.cuda.synchronize()
+            dist.barrier()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            for _ in range(reps):
+                g.replay()
+            e1.record()
+            e1.synchronize()
+            t = dist.max(e0.elapsed_time(e1) * 1e-3 / (reps * n))
+            napp_mid = max(1, -(-warmup // n)) + (reps - 1) / 2.0
+            return t, n, reps, napp_mid, n * rows_bytes
+
+        packed_bytes = env["info"].total_rows * 512
+        t, n, reps, napp_mid, span = timed(env["plan"], env["Kc"], env["Vc"], packed_bytes)
+        rows = kept + wl.L * NHl * (napp_mid + 1)
+        algo = step_bytes(wl, rows)
+        res = {"us_per_step": round(t * 1e6, 2), "gb_per_step": round(algo / 1e9, 5),
+               "gbs": round(algo / t / 1e9, 1), "frac_of_hbm": round(algo / t / 1e9 / peak, 4),
+               "steps": reps * n,
+               "l2": "rotating %d copies of the packed caches, %.0f MB in all (%.1f x the %.0f MB L2)"
+                     % (n, span / 1e6, span / l2, l2 / 1e6)}
+        dense = dkv.dkv_plan_dense(env["Tc"], env["shape"], T_stride=env["T_stride"])
+        td, dn, _, dmid, dspan = timed(dense, env["K"], env["V"], env["K"].numel() * 4)
+        dense.close()
+        drows = wl.L * wl.Hkv * float(env["Tc"].sum()) + wl.L * NHl * (dmid + 1)
+        res.update({"dense_us_per_step": round(td * 1e6, 2), "dense_gbs": round(step_bytes(wl, drows) / td / 1e9, 1),
+                    "dense_l2": "rotating %d copies of the dense caches, %.0f MB" % (dn, dspan / 1e6),
+                    "speedup_of_compacted": round(td / t, 3), "ideal_speedup": round(drows / rows, 3)})
+        return res
+    finally:
+        env["plan"].close()
+        del env
+        torch.cuda.empty_cache()
 
 
 def time_graph(runner, steps, warmup, dist, clocks=None):
@@ -767,6 +892,20 @@ def run_dkv(args, dist):
     st = dkv.dkv_plan_status(env["plan"])
     res["device_status_word"] = st
     env["plan"].close()
+    del env
+    torch.cuda.empty_cache()
+    if not args.profile and not args.no_workloads:
+        # The other workloads of the benchmark set that fit a few seconds: the
+        # 32K Llama cache and the 64K Qwen cache (35 % budget), and the 1-layer
+        # 4K case measured from HBM over rotated copies.
+        wls = {}
+        for name in ("llama8b-32k", "qwen7b-64k-b4-r35"):
+            if name != wl.name:
+                with nvtx(f"workload {name} (timed)"):
+                    wls[name] = workload_line(name, dev, steps, warmup, dist, peak)
+        with nvtx("workload llama8b-1layer-4k, rotated caches (timed)"):
+            wls["llama8b-1layer-4k"] = rotated_small_workload("llama8b-1layer-4k", dev, steps, warmup, dist, peak)
+        res["workloads"] = wls
     return res
 
 

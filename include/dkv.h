@@ -99,8 +99,12 @@ const char* dkv_last_error(void);
  * H % H_kv != 0, head_dim != 128, a negative length or reserve, B out of range,
  * or a layer whose rows (with reserve) exceed 2^31 - 1; DKV_ERR_RANGE when some
  * Tc[b] - S - R > D * W (positions with no bin); DKV_ERR_OOM / DKV_ERR_CUDA.
- * Synchronises `stream`: once to learn the total row count, and before it
- * returns (the map's temporaries are then freed).
+ * Synchronises `stream` once, to learn the row counts (which size the index
+ * list and the caller's packed caches). The index list is then written by a
+ * kernel that the call leaves running on `stream`: work queued on `stream`
+ * afterwards is ordered after it; other streams must wait for `stream`.
+ * Device memory: one allocation for the plan's metadata and counters, and one,
+ * sized after the sync, for the index list and the split-K workspace.
  */
 dkv_status dkv_map_pattern(const uint8_t* M_host, const int32_t* ctx_len_host, int32_t B,
                            const dkv_shape* s, int32_t reserve_rows, cudaStream_t stream,

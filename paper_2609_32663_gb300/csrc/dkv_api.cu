@@ -24,6 +24,8 @@ struct dkv_plan {
     int64_t total_rows = 0;   // rows of the packed (or dense) cache
     int64_t kept_rows = 0;
     int device = 0;
+    void* d_arena = nullptr;    // one allocation: the map's metadata and counters (the workspace too, dense plans)
+    void* d_arena2 = nullptr;   // map plans: the index list and the workspace, sized after the map's one sync
     int32_t* d_len = nullptr;   // [NH]
     int64_t* d_off = nullptr;   // [NH+1]
     int64_t* d_ioff = nullptr;  // [NH+1]
@@ -31,12 +33,13 @@ struct dkv_plan {
     int32_t* d_status = nullptr;
     float* d_work = nullptr;    // split-K partials
     int32_t* d_slab_count = nullptr;  // [B*H_kv][cols][2] arrival / written counters of the fused combine
-    dkv::DecodeConfig cfg{};        // the decode step's kernel
+    dkv::DecodeConfig cfg{};         // the decode step's kernel (cfg_f32 or cfg_mma)
+    dkv::DecodeConfig cfg_f32{};     // fp32 kernel (caches of 2^31 rows or more)
+    dkv::DecodeConfig cfg_mma{};     // tensor-core kernel of the decode step
     dkv::DecodeConfig cfg_multi1{};  // multi-query, one column tile (tensor-core plans)
     dkv::DecodeConfig cfg_multi{};   // multi-query, two column tiles (tensor-core plans)
-    int64_t slots = 0;              // (CTA, slab) partial slots: CTAs + slabs of a layer
-    dkv::WorkspaceLayout work{};    // carve-up of d_work
-    int nctas_cap = 0, warps_cap = 0, cols_cap = 0;  // workspace sized for these
+    dkv::WorkspaceLayout work{};     // carve-up of d_work
+    int cols_cap = 0;                // columns the workspace and counters are sized for
     int use_mma = 0;  // tensor-core decode kernel (needs the cache's row count for its tensor maps)
     int64_t inplace_stride = 0;  // > 0: slab h lives at rows h * stride of the dense buffer (in place)
     int32_t* d_order = nullptr;  // in place: [NH] slabs by length, longest first, then a claim counter
@@ -111,14 +114,8 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 void release(dkv_plan* p)
 {
     if (!p) return;
-    cudaFree(p->d_len);
-    cudaFree(p->d_off);
-    cudaFree(p->d_ioff);
-    cudaFree(p->d_idx);
-    cudaFree(p->d_status);
-    cudaFree(p->d_work);
-    cudaFree(p->d_slab_count);
-    cudaFree(p->d_order);
+    cudaFree(p->d_arena);
+    cudaFree(p->d_arena2);
     delete p;
 }
 
@@ -140,44 +137,72 @@ dkv_status check_shape(const dkv_shape* s, int32_t B)
     return DKV_OK;
 }
 
-// Split-K workspace and decode launch configuration of a finished plan.
-dkv_status finish_plan(dkv_plan* p)
+// Byte offsets of the plan's device arrays inside its one allocation, each on a
+// 256-byte boundary.
+struct ArenaLayout {
+    size_t bytes = 0;
+    template <class T>
+    size_t take(size_t count)
+    {
+        const size_t off = (bytes + 255) / 256 * 256;
+        bytes = off + std::max<size_t>(count, 1) * sizeof(T);
+        return off;
+    }
+};
+
+template <class T>
+T* at(void* base, size_t off)
+{
+    return reinterpret_cast<T*>(static_cast<unsigned char*>(base) + off);
+}
+
+// Launch configurations of every decode kernel a plan may run (host queries,
+// no device work), and the split-K workspace that serves all of them: slots for
+// the largest grid plus the slabs of a layer, warp records for the largest grid
+// x warps, kMaxCols columns.
+dkv_status plan_configs(dkv_plan* p)
 {
     cudaGetDevice(&p->device);
-    p->use_mma = p->total_rows >= 1 && p->total_rows <= dkv::kMaxMmaRows;
     cudaError_t e;
-    if (p->use_mma) {
-        const int NHl = p->B * p->s.H_kv;
-        std::vector<int32_t> len((size_t)p->s.L * NHl);
-        if ((e = cudaMemcpy(len.data(), p->d_len, sizeof(int32_t) * len.size(), cudaMemcpyDeviceToHost)) != cudaSuccess)
-            return cuda_fail(e, "read lengths");
-        p->layer_rows.assign((size_t)p->s.L, 0);
-        for (size_t h = 0; h < len.size(); ++h) p->layer_rows[h / NHl] += len[h];
-        if ((e = dkv::decode_config_mma(p->G, p->B, 0, &p->cfg)) != cudaSuccess) return cuda_fail(e, "decode_config");
-        if ((e = dkv::decode_config_mma(p->G, p->B, 1, &p->cfg_multi1)) != cudaSuccess ||
-            (e = dkv::decode_config_mma(p->G, p->B, 2, &p->cfg_multi)) != cudaSuccess)
-            return cuda_fail(e, "decode_config (multi-query)");
-        p->nctas_cap = std::max({p->cfg.nctas, p->cfg_multi1.nctas, p->cfg_multi.nctas});
-        p->warps_cap = std::max({p->cfg.nwarps, p->cfg_multi1.nwarps, p->cfg_multi.nwarps});
-        p->cols_cap = dkv::kMaxCols;
-    } else {
-        if ((e = dkv::decode_config(p->G, p->B, &p->cfg)) != cudaSuccess) return cuda_fail(e, "decode_config");
-        p->nctas_cap = p->cfg.nctas;
-        p->warps_cap = p->cfg.nwarps;
-        p->cols_cap = p->G;
+    if ((e = dkv::decode_config(p->G, p->B, &p->cfg_f32)) != cudaSuccess) return cuda_fail(e, "decode_config");
+    if ((e = dkv::decode_config_mma(p->G, p->B, 0, &p->cfg_mma)) != cudaSuccess ||
+        (e = dkv::decode_config_mma(p->G, p->B, 1, &p->cfg_multi1)) != cudaSuccess ||
+        (e = dkv::decode_config_mma(p->G, p->B, 2, &p->cfg_multi)) != cudaSuccess)
+        return cuda_fail(e, "decode_config (tensor cores)");
+    int64_t ctas = 0, warp_records = 0;
+    for (const dkv::DecodeConfig* c : {&p->cfg_f32, &p->cfg_mma, &p->cfg_multi1, &p->cfg_multi}) {
+        ctas = std::max<int64_t>(ctas, c->nctas);
+        warp_records = std::max<int64_t>(warp_records, (int64_t)c->nctas * c->nwarps);
     }
-    p->slots = (int64_t)p->nctas_cap + p->B * p->s.H_kv;
-    p->work = dkv::decode_workspace(p->nctas_cap, p->warps_cap, p->cols_cap, p->B * p->s.H_kv);
-    dkv_status st = dalloc(&p->d_work, (size_t)p->work.total, "split-K workspace");
-    if (st != DKV_OK) return st;
-    st = dalloc(&p->d_status, 1, "status word");
-    if (st != DKV_OK) return st;
-    if ((e = cudaMemset(p->d_status, 0, sizeof(int32_t))) != cudaSuccess) return cuda_fail(e, "cudaMemset");
-    st = dalloc(&p->d_slab_count, (size_t)2 * p->B * p->s.H_kv * p->cols_cap, "slab counters");
-    if (st != DKV_OK) return st;
-    if ((e = cudaMemset(p->d_slab_count, 0, sizeof(int32_t) * 2 * p->B * p->s.H_kv * p->cols_cap)) != cudaSuccess)
-        return cuda_fail(e, "cudaMemset");
+    p->cols_cap = dkv::kMaxCols;
+    p->work = dkv::workspace_layout(ctas + (int64_t)p->B * p->s.H_kv, warp_records, p->cols_cap);
     return DKV_OK;
+}
+
+// Places the counters (status word, then the fused combine's slab counters) as
+// one int32 block that a single memset zeroes, and the split-K workspace.
+struct ZeroBlock {
+    size_t off = 0, count = 0;
+};
+ZeroBlock take_zeroed(ArenaLayout& lay, const dkv_plan* p, size_t extra)
+{
+    ZeroBlock z;
+    z.count = 1 + (size_t)2 * p->B * p->s.H_kv * p->cols_cap + extra;
+    z.off = lay.take<int32_t>(z.count);
+    return z;
+}
+
+void place_zeroed(dkv_plan* p, const ZeroBlock& z)
+{
+    p->d_status = at<int32_t>(p->d_arena, z.off);
+    p->d_slab_count = p->d_status + 1;
+}
+
+// The decode kernel of a plan whose row count is known.
+void choose_kernel(dkv_plan* p)
+{
+    p->use_mma = p->total_rows >= 1 && p->total_rows <= dkv::kMaxMmaRows;
+    p->cfg = p->use_mma ? p->cfg_mma : p->cfg_f32;
 }
 
 }  // namespace
@@ -204,6 +229,14 @@ const char* dkv_last_error(void) { return g_err; }
 
 // The map of dkv_map_pattern and dkv_map_pattern_inplace: slab offsets are the
 // running sum of (len + reserve), or h * inplace_stride when that is > 0.
+//
+// Device work, all on `stream`: one allocation for the plan's metadata and
+// counters (the map's inputs M and Tc live there too), one memset of the
+// counters, the copies of M and Tc, the runs kernel (and, in place, the slab
+// order), one read of the totals -- the only synchronisation -- then a second
+// allocation, sized by the totals, for the index list and the split-K
+// workspace, and the index list's write. The call returns without waiting for
+// the write: later calls on `stream` are ordered after it.
 static dkv_status map_pattern_impl(const uint8_t* M_host, const int32_t* ctx_len_host, int32_t B,
                                    const dkv_shape* s, int32_t reserve_rows, int64_t inplace_stride,
                                    cudaStream_t stream, dkv_plan** out)
@@ -238,6 +271,9 @@ static dkv_status map_pattern_impl(const uint8_t* M_host, const int32_t* ctx_len
         if (layer_rows > 0x7fffffffLL)
             return fail(DKV_ERR_INVALID_ARG, "a layer would hold %lld rows (> 2^31-1)", (long long)layer_rows);
     }
+    const int64_t NH64 = (int64_t)s->L * B * s->H_kv;
+    if (NH64 > 0x7fffffffLL) return fail(DKV_ERR_INVALID_ARG, "L*B*H_kv=%lld slabs (> 2^31-1)", (long long)NH64);
+    const int NH = (int)NH64;
 
     dkv_plan* p = new (std::nothrow) dkv_plan();
     if (!p) return fail(DKV_ERR_OOM, "host allocation of the plan failed");
@@ -247,50 +283,49 @@ static dkv_status map_pattern_impl(const uint8_t* M_host, const int32_t* ctx_len
     p->reserve = reserve_rows;
     p->inplace_stride = inplace_stride;
     p->T_stride = inplace_stride;
-
-    const int NH = s->L * B * s->H_kv;
-    const int nchunks = Tmax > 0 ? (Tmax + dkv::kMapChunk - 1) / dkv::kMapChunk : 1;
-    uint8_t *dM = nullptr, *dU = nullptr;
-    int32_t *dTc = nullptr, *dcnt = nullptr;
-    std::vector<int64_t> tail(2);
-    auto cleanup = [&]() {
-        cudaFree(dM);
-        cudaFree(dU);
-        cudaFree(dTc);
-        cudaFree(dcnt);
+    auto bail = [&](dkv_status e) {
+        release(p);
+        return e;
     };
-    if ((st = dalloc(&dM, nM, "pattern")) != DKV_OK ||
-        (st = dalloc(&dU, (size_t)s->L * s->H_kv * s->D, "union pattern")) != DKV_OK ||
-        (st = dalloc(&dTc, (size_t)B, "context lengths")) != DKV_OK ||
-        (st = dalloc(&dcnt, (size_t)NH * nchunks, "chunk counts")) != DKV_OK ||
-        (st = dalloc(&p->d_len, (size_t)NH, "lengths")) != DKV_OK ||
-        (st = dalloc(&p->d_off, (size_t)NH + 1, "offsets")) != DKV_OK ||
-        (st = dalloc(&p->d_ioff, (size_t)NH + 1, "index offsets")) != DKV_OK) {
-        cleanup();
-        release(p);
-        return st;
-    }
+    p->cols_cap = dkv::kMaxCols;
+
+    ArenaLayout lay;
+    const size_t o_len = lay.take<int32_t>((size_t)NH), o_off = lay.take<int64_t>((size_t)NH + 1),
+                 o_ioff = lay.take<int64_t>((size_t)NH + 1), o_nruns = lay.take<int32_t>((size_t)NH),
+                 o_runs = lay.take<int2>((size_t)NH * (s->D + 2)), o_tail = lay.take<int64_t>((size_t)3 + s->L),
+                 o_M = lay.take<uint8_t>(nM), o_Tc = lay.take<int32_t>((size_t)B),
+                 o_order = inplace_stride > 0 ? lay.take<int32_t>((size_t)NH + 1) : 0;
+    const ZeroBlock zb = take_zeroed(lay, p, 1);  // + the runs kernel's CTA counter
+    if ((st = dalloc(reinterpret_cast<unsigned char**>(&p->d_arena), lay.bytes, "plan metadata")) != DKV_OK)
+        return bail(st);
+    p->d_len = at<int32_t>(p->d_arena, o_len);
+    p->d_off = at<int64_t>(p->d_arena, o_off);
+    p->d_ioff = at<int64_t>(p->d_arena, o_ioff);
+    p->d_order = inplace_stride > 0 ? at<int32_t>(p->d_arena, o_order) : nullptr;
+    place_zeroed(p, zb);
+
     cudaError_t e;
-    if (nM && (e = cudaMemcpyAsync(dM, M_host, nM, cudaMemcpyHostToDevice, stream)) != cudaSuccess) {
-        cleanup();
-        release(p);
-        return cuda_fail(e, "copy pattern");
-    }
-    if ((e = cudaMemcpyAsync(dTc, ctx_len_host, (size_t)B * 4, cudaMemcpyHostToDevice, stream)) != cudaSuccess) {
-        cleanup();
-        release(p);
-        return cuda_fail(e, "copy ctx_len");
-    }
-    // Pass A: union, counts, scan (idx is allocated once its size is known).
+    if ((e = cudaMemsetAsync(p->d_status, 0, zb.count * sizeof(int32_t), stream)) != cudaSuccess)
+        return bail(cuda_fail(e, "clear counters"));
+    if (nM && (e = cudaMemcpyAsync(at<uint8_t>(p->d_arena, o_M), M_host, nM, cudaMemcpyHostToDevice, stream)) !=
+                  cudaSuccess)
+        return bail(cuda_fail(e, "copy pattern"));
+    if ((e = cudaMemcpyAsync(at<int32_t>(p->d_arena, o_Tc), ctx_len_host, (size_t)B * 4, cudaMemcpyHostToDevice,
+                             stream)) != cudaSuccess)
+        return bail(cuda_fail(e, "copy ctx_len"));
+
     dkv::MapArgs ma{};
-    ma.M = dM;
-    ma.U = dU;
-    ma.Tc = dTc;
-    ma.chunk_cnt = dcnt;
+    ma.M = at<uint8_t>(p->d_arena, o_M);
+    ma.Tc = at<int32_t>(p->d_arena, o_Tc);
+    ma.runs = at<int2>(p->d_arena, o_runs);
+    ma.nruns = at<int32_t>(p->d_arena, o_nruns);
     ma.len = p->d_len;
     ma.off = p->d_off;
     ma.ioff = p->d_ioff;
     ma.idx = nullptr;
+    ma.tail = at<int64_t>(p->d_arena, o_tail);
+    ma.done = reinterpret_cast<unsigned*>(p->d_status + zb.count - 1);
+    ma.order = p->d_order;
     ma.L = s->L;
     ma.H = s->H;
     ma.Hkv = s->H_kv;
@@ -300,64 +335,30 @@ static dkv_status map_pattern_impl(const uint8_t* M_host, const int32_t* ctx_len
     ma.recent = s->recent;
     ma.bin_width = s->bin_width;
     ma.reserve = reserve_rows;
-    ma.nchunks = nchunks;
     ma.NH = NH;
     ma.stride = inplace_stride;
-    if ((st = launched(dkv::launch_map(ma, stream), "map kernels")) != DKV_OK) {
-        cleanup();
-        release(p);
-        return st;
-    }
-    // The one synchronisation: learn total and kept row counts.
-    if ((e = cudaMemcpyAsync(&tail[0], p->d_off + NH, 8, cudaMemcpyDeviceToHost, stream)) != cudaSuccess ||
-        (e = cudaMemcpyAsync(&tail[1], p->d_ioff + NH, 8, cudaMemcpyDeviceToHost, stream)) != cudaSuccess ||
-        (e = cudaStreamSynchronize(stream)) != cudaSuccess) {
-        cleanup();
-        release(p);
-        return cuda_fail(e, "map: read totals");
-    }
+    if ((st = launched(dkv::launch_map(ma, stream), "map kernels")) != DKV_OK) return bail(st);
+    // The one synchronisation: the totals (rows, kept rows, longest slab, rows of each layer).
+    std::vector<int64_t> tail((size_t)3 + s->L);
+    if ((e = cudaMemcpyAsync(tail.data(), ma.tail, sizeof(int64_t) * tail.size(), cudaMemcpyDeviceToHost, stream)) !=
+            cudaSuccess ||
+        (e = cudaStreamSynchronize(stream)) != cudaSuccess)
+        return bail(cuda_fail(e, "map: read totals"));
     p->total_rows = tail[0];
     p->kept_rows = tail[1];
-    if ((st = dalloc(&p->d_idx, (size_t)p->kept_rows, "kept index list")) != DKV_OK) {
-        cleanup();
-        release(p);
-        return st;
-    }
+    p->layer_rows.assign(tail.begin() + 3, tail.end());
+    if ((st = plan_configs(p)) != DKV_OK) return bail(st);
+    ArenaLayout lay2;
+    const size_t o_idx = lay2.take<int32_t>((size_t)p->kept_rows), o_work = lay2.take<float>((size_t)p->work.total);
+    if ((st = dalloc(reinterpret_cast<unsigned char**>(&p->d_arena2), lay2.bytes, "index list and workspace")) !=
+        DKV_OK)
+        return bail(st);
+    p->d_idx = at<int32_t>(p->d_arena2, o_idx);
+    p->d_work = at<float>(p->d_arena2, o_work);
     ma.idx = p->d_idx;
-    if ((st = launched(dkv::launch_map_write(ma, stream), "map write kernel")) != DKV_OK) {
-        cleanup();
-        release(p);
-        return st;
-    }
-    if ((e = cudaStreamSynchronize(stream)) != cudaSuccess) {
-        cleanup();
-        release(p);
-        return cuda_fail(e, "map: kernels");
-    }
-    cleanup();
-    if (inplace_stride > 0) {
-        // The in-place compaction streams whole slabs, longest first.
-        std::vector<int32_t> len((size_t)NH), order((size_t)NH + 1, 0);
-        if ((e = cudaMemcpy(len.data(), p->d_len, sizeof(int32_t) * NH, cudaMemcpyDeviceToHost)) != cudaSuccess) {
-            release(p);
-            return cuda_fail(e, "map: read lengths");
-        }
-        for (int h = 0; h < NH; ++h) order[(size_t)h] = h;
-        std::stable_sort(order.begin(), order.begin() + NH, [&](int32_t x, int32_t y) { return len[x] > len[y]; });
-        if ((st = dalloc(&p->d_order, (size_t)NH + 1, "slab order")) != DKV_OK) {
-            release(p);
-            return st;
-        }
-        if ((e = cudaMemcpy(p->d_order, order.data(), sizeof(int32_t) * (NH + 1), cudaMemcpyHostToDevice)) !=
-            cudaSuccess) {
-            release(p);
-            return cuda_fail(e, "map: slab order");
-        }
-    }
-    if ((st = finish_plan(p)) != DKV_OK) {
-        release(p);
-        return st;
-    }
+    if ((st = launched(dkv::launch_map_write(ma, (int)tail[2], stream), "map write kernel")) != DKV_OK)
+        return bail(st);
+    choose_kernel(p);
     *out = p;
     return ok();
 }
@@ -402,6 +403,13 @@ dkv_status dkv_plan_dense(const int32_t* ctx_len_host, int32_t B, const dkv_shap
     p->dense = 1;
     p->T_stride = T_stride;
     p->reserve = (int)(T_stride - Tmax);
+    auto bail = [&](dkv_status e) {
+        release(p);
+        return e;
+    };
+    if ((st = plan_configs(p)) != DKV_OK) return bail(st);
+    // The uncompressed layout is given by the arguments: slab h holds the
+    // sequence's Tc[b] rows at row h * T_stride.
     const int NH = s->L * B * s->H_kv;
     std::vector<int32_t> len(NH);
     std::vector<int64_t> off(NH + 1), ioff(NH + 1);
@@ -417,24 +425,28 @@ dkv_status dkv_plan_dense(const int32_t* ctx_len_host, int32_t B, const dkv_shap
     ioff[NH] = run;
     p->total_rows = off[NH];
     p->kept_rows = run;
+    p->layer_rows.assign((size_t)s->L, 0);
+    for (int h = 0; h < NH; ++h) p->layer_rows[(size_t)h / (B * s->H_kv)] += len[h];
+    ArenaLayout lay;
+    const size_t o_len = lay.take<int32_t>((size_t)NH), o_off = lay.take<int64_t>((size_t)NH + 1),
+                 o_ioff = lay.take<int64_t>((size_t)NH + 1);
+    const ZeroBlock zb = take_zeroed(lay, p, 0);
+    const size_t o_work = lay.take<float>((size_t)p->work.total);
+    if ((st = dalloc(reinterpret_cast<unsigned char**>(&p->d_arena), lay.bytes, "plan metadata")) != DKV_OK)
+        return bail(st);
+    p->d_len = at<int32_t>(p->d_arena, o_len);
+    p->d_off = at<int64_t>(p->d_arena, o_off);
+    p->d_ioff = at<int64_t>(p->d_arena, o_ioff);
+    p->d_work = at<float>(p->d_arena, o_work);
+    place_zeroed(p, zb);
     cudaError_t e;
-    if ((st = dalloc(&p->d_len, (size_t)NH, "lengths")) != DKV_OK ||
-        (st = dalloc(&p->d_off, (size_t)NH + 1, "offsets")) != DKV_OK ||
-        (st = dalloc(&p->d_ioff, (size_t)NH + 1, "row prefix")) != DKV_OK) {
-        release(p);
-        return st;
-    }
-    if ((e = cudaMemcpyAsync(p->d_len, len.data(), (size_t)NH * 4, cudaMemcpyHostToDevice, stream)) != cudaSuccess ||
+    if ((e = cudaMemsetAsync(p->d_status, 0, zb.count * sizeof(int32_t), stream)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(p->d_len, len.data(), (size_t)NH * 4, cudaMemcpyHostToDevice, stream)) != cudaSuccess ||
         (e = cudaMemcpyAsync(p->d_off, off.data(), (size_t)(NH + 1) * 8, cudaMemcpyHostToDevice, stream)) != cudaSuccess ||
         (e = cudaMemcpyAsync(p->d_ioff, ioff.data(), (size_t)(NH + 1) * 8, cudaMemcpyHostToDevice, stream)) != cudaSuccess ||
-        (e = cudaStreamSynchronize(stream)) != cudaSuccess) {
-        release(p);
-        return cuda_fail(e, "dense plan upload");
-    }
-    if ((st = finish_plan(p)) != DKV_OK) {
-        release(p);
-        return st;
-    }
+        (e = cudaStreamSynchronize(stream)) != cudaSuccess)
+        return bail(cuda_fail(e, "dense plan upload"));
+    choose_kernel(p);
     *out = p;
     return ok();
 }

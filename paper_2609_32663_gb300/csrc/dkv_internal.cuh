@@ -14,23 +14,27 @@ constexpr int kRowBytes = 256;  // bytes per bf16 row
 // ---------------------------------------------------------------- pattern map
 struct MapArgs {
     const uint8_t* M;       // [L][H][D]
-    uint8_t* U;             // [L][Hkv][D], union over each GQA group
     const int32_t* Tc;      // [B]
-    int32_t* chunk_cnt;     // [NH][nchunks], kept count of each position chunk
+    int2* runs;             // [NH][D+2]: kept runs of each slab in token order, (first output row, first position)
+    int32_t* nruns;         // [NH]
     int32_t* len;           // [NH]
     int64_t* off;           // [NH+1]
     int64_t* ioff;          // [NH+1]
     int32_t* idx;           // [kept]
+    int64_t* tail;          // [3 + L]: total rows, kept rows, longest slab, kept rows of each layer
+    unsigned* done;         // CTAs of the runs pass that have finished (zero before the launch)
+    int32_t* order;         // in place: [NH] slabs by length, longest first; else null
     int L, H, Hkv, D, B, sink, recent, bin_width, reserve;
-    int nchunks;            // position chunks per slab
     int NH;                 // L*B*Hkv
     int64_t stride;         // 0: slabs packed end to end; > 0: slab h starts at row h * stride (in place)
 };
-constexpr int kMapChunk = 8192;  // positions per CTA in the count/write passes
+constexpr int kMapChunk = 8192;  // output rows per CTA of the index-list write
 
-// Union, per-chunk counts and the offset scan; then, once idx is allocated, the writes.
+// The runs of every slab, their lengths, the offset scans and the totals (and,
+// in place, the slab order); then, once idx is allocated, the index-list write
+// (max_len: the longest slab, from the totals).
 cudaError_t launch_map(const MapArgs& a, cudaStream_t st);
-cudaError_t launch_map_write(const MapArgs& a, cudaStream_t st);
+cudaError_t launch_map_write(const MapArgs& a, int max_len, cudaStream_t st);
 
 // ---------------------------------------------------------------- compaction
 struct CompactArgs {

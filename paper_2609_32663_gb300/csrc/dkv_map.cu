@@ -1,162 +1,223 @@
 // Pattern -> positions map (Sec. 3.4, Eqs. 4-5 and the GQA union).
 //
-// Four stream-ordered kernels, no device-wide waits:
-//   union_kernel   U[l][g][d] = OR_j M[l][g*G + j][d]       (GQA union of bins)
-//   count_kernel   per (slab, chunk of 8192 positions): kept count via warp ballot
-//   scan_kernel    one CTA: per-slab lengths, chunk bases, slab offsets (int64)
-//   write_kernel   recomputes the keep bits, ballot + popc + CTA scan -> idx
-// keep(p) = p < S  or  p >= Tc - R  or  U[l][g][(Tc - R - 1 - p) / W].
+// keep(p) = p < S  or  p >= Tc - R  or  U[l][g][(Tc - R - 1 - p) / W],  with
+// U[l][g][d] = OR_j M[l][g G + j][d]. Between the sink and the recent window the
+// decision is constant over the W positions of a distance bin, so a slab's kept
+// positions are a few runs of consecutive positions: the sink, each kept bin the
+// context reaches (far bins first: token order), the recent window. The map is
+// built per bin instead of per position:
+//
+//   runs_kernel   one warp per slab (layer, sequence, KV head). Lanes take 32
+//                 bins at a time in token order: the GQA union of the bin's query
+//                 heads, its positions clipped to the context, a warp ballot over
+//                 the kept bins and a prefix scan of their lengths, which place
+//                 each kept bin's run (first output row, first position) in the
+//                 slab's run list and give the slab's length. The last CTA to
+//                 finish scans the lengths over the flat slab order into slab
+//                 offsets (len + reserve, or h * stride in place), index offsets,
+//                 and the totals the host reads (rows, kept rows, longest slab,
+//                 kept rows per layer).
+//   order_kernel  (in place only) the slabs by length, longest first, ties by
+//                 index: slab h goes to its rank among all slabs.
+//   write_kernel  one CTA per (slab, kMapChunk output rows): output row r of slab h
+//                 is the position runs[i].pos + (r - runs[i].row) of the run i
+//                 holding r; lanes take consecutive rows, so the index list is
+//                 written with coalesced stores, and no position is visited
+//                 twice. Dropped positions are never touched.
 #include "dkv_internal.cuh"
 
 namespace dkv {
 namespace {
 
-__global__ void union_kernel(const uint8_t* __restrict__ M, uint8_t* __restrict__ U, int L, int H,
-                             int Hkv, int D)
+constexpr unsigned kFullMask = 0xffffffffu;
+constexpr int kRunsThreads = 256;  // 8 slabs per CTA, one a warp
+constexpr int kWriteThreads = 256;
+
+__global__ void __launch_bounds__(kRunsThreads) runs_kernel(const MapArgs a)
 {
-    const int G = H / Hkv;
-    const int64_t n = (int64_t)L * Hkv * D;
-    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
-         i += (int64_t)gridDim.x * blockDim.x) {
-        const int d = (int)(i % D);
-        const int64_t lg = i / D;  // l*Hkv + g
-        const uint8_t* row = M + (lg * G) * D + d;
-        uint8_t u = 0;
-        for (int j = 0; j < G; ++j) u |= row[(int64_t)j * D];
-        U[i] = u;
-    }
-}
-
-// Retention decision of KV head slab (layer, g) at position p of a Tc-token context.
-__device__ __forceinline__ bool keep_pos(const uint8_t* __restrict__ Urow, int p, int Tc, int S,
-                                         int R, int W)
-{
-    if (p < S || p >= Tc - R) return true;
-    return Urow[(Tc - R - 1 - p) / W] != 0;
-}
-
-struct SlabView {
-    const uint8_t* Urow;
-    int Tc;
-};
-
-__device__ __forceinline__ SlabView slab_view(const MapArgs& a, int h)
-{
-    const int g = h % a.Hkv;
-    const int b = (h / a.Hkv) % a.B;
-    const int l = h / (a.Hkv * a.B);
-    return SlabView{a.U + ((int64_t)l * a.Hkv + g) * a.D, a.Tc[b]};
-}
-
-constexpr int kMapThreads = 256;
-constexpr int kMapIters = kMapChunk / kMapThreads;  // 32 positions per thread
-
-__global__ void __launch_bounds__(kMapThreads) count_kernel(const MapArgs a)
-{
-    const int h = blockIdx.x, c = blockIdx.y;
-    const SlabView v = slab_view(a, h);
-    const int base = c * kMapChunk;
-    int cnt = 0;
-    if (base < v.Tc) {
-        for (int k = 0; k < kMapIters; ++k) {
-            const int p = base + k * kMapThreads + threadIdx.x;
-            const bool kp = p < v.Tc && keep_pos(v.Urow, p, v.Tc, a.sink, a.recent, a.bin_width);
-            const unsigned bal = __ballot_sync(0xffffffffu, kp);
-            cnt += __popc(bal);  // identical in every lane of the warp
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int h = blockIdx.x * (kRunsThreads / 32) + warp;
+    if (h < a.NH) {
+        const int g = h % a.Hkv;
+        const int b = (h / a.Hkv) % a.B;
+        const int l = h / (a.Hkv * a.B);
+        const int G = a.H / a.Hkv;
+        const int Tc = a.Tc[b];
+        const int S = a.sink, R = a.recent, W = a.bin_width;
+        int2* run = a.runs + (int64_t)h * (a.D + 2);
+        int n = 0, out = 0;
+        if (Tc <= S + R) {
+            // Sink and recent window cover the whole context: one run.
+            if (Tc > 0) {
+                if (lane == 0) run[0] = make_int2(0, 0);
+                n = 1;
+            }
+            out = Tc;
+        } else {
+            const int C = Tc - S - R;          // positions between sink and recent window
+            const int nb = (int)(((int64_t)C + W - 1) / W);  // bins the context reaches (<= D: checked on the host)
+            if (lane == 0) run[0] = make_int2(0, 0);  // the sink
+            n = 1;
+            out = S;
+            const uint8_t* Mg = a.M + ((int64_t)l * a.H + (int64_t)g * G) * a.D;
+            for (int k0 = 0; k0 < nb; k0 += 32) {
+                const int k = k0 + lane;  // k-th bin in token order: d = nb - 1 - k
+                bool on = false;
+                int len = 0, lo = 0;
+                if (k < nb) {
+                    const int d = nb - 1 - k;
+                    uint8_t u = 0;
+                    for (int j = 0; j < G; ++j) u |= __ldg(Mg + (int64_t)j * a.D + d);
+                    on = u != 0;
+                    len = min(W, C - d * W);                  // positions of bin d inside the context
+                    lo = (int)max((int64_t)S, (int64_t)Tc - R - (int64_t)(d + 1) * W);  // its first position
+                }
+                const unsigned kept = __ballot_sync(kFullMask, on);
+                int incl = on ? len : 0;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    const int v = __shfl_up_sync(kFullMask, incl, o);
+                    if (lane >= o) incl += v;
+                }
+                if (on) {
+                    const int rank = __popc(kept & ((1u << lane) - 1u));
+                    run[n + rank] = make_int2(out + incl - len, lo);
+                }
+                n += __popc(kept);
+                out += __shfl_sync(kFullMask, incl, 31);
+            }
+            if (lane == 0) run[n] = make_int2(out, Tc - R);  // the recent window
+            n += 1;
+            out += R;
+        }
+        if (lane == 0) {
+            a.len[h] = out;
+            a.nruns[h] = n;
         }
     }
-    __shared__ int warp_cnt[kMapThreads / 32];
-    if ((threadIdx.x & 31) == 0) warp_cnt[threadIdx.x >> 5] = cnt;
+
+    // The last CTA to finish scans the slab lengths.
+    __shared__ bool last;
     __syncthreads();
     if (threadIdx.x == 0) {
-        int s = 0;
-        for (int w = 0; w < kMapThreads / 32; ++w) s += warp_cnt[w];
-        a.chunk_cnt[(int64_t)h * a.nchunks + c] = s;
-    }
-}
-
-// One CTA. Pass 1: slab lengths, and chunk counts turned into exclusive chunk
-// bases in place. Pass 2: exclusive scans of len+reserve (off) and len (ioff)
-// over the flat slab order, as a CTA-wide scan of per-thread partial sums.
-constexpr int kScanThreads = 1024;
-
-__global__ void __launch_bounds__(kScanThreads) scan_kernel(const MapArgs a)
-{
-    for (int h = threadIdx.x; h < a.NH; h += kScanThreads) {
-        int32_t* cc = a.chunk_cnt + (int64_t)h * a.nchunks;
-        int s = 0;
-        for (int c = 0; c < a.nchunks; ++c) {
-            const int n = cc[c];
-            cc[c] = s;
-            s += n;
-        }
-        a.len[h] = s;
+        __threadfence();
+        last = atomicAdd(a.done, 1u) == gridDim.x - 1;
     }
     __syncthreads();
-
-    const int per = (a.NH + kScanThreads - 1) / kScanThreads;
-    const int h0 = min(a.NH, (int)threadIdx.x * per);
-    const int h1 = min(a.NH, h0 + per);
+    if (!last) return;
+    __threadfence();
+    constexpr int T = kRunsThreads;
+    const int per = (a.NH + T - 1) / T;
+    const int h0 = min(a.NH, (int)threadIdx.x * per), h1 = min(a.NH, h0 + per);
     int64_t s_off = 0, s_ioff = 0;
+    int mx = 0;
     for (int h = h0; h < h1; ++h) {
-        s_off += (int64_t)a.len[h] + a.reserve;
-        s_ioff += a.len[h];
+        const int n = __ldcg(a.len + h);
+        s_off += (int64_t)n + a.reserve;
+        s_ioff += n;
+        mx = max(mx, n);
     }
-    __shared__ int64_t sh_off[kScanThreads], sh_ioff[kScanThreads];
+    __shared__ int64_t sh_off[T], sh_ioff[T];
+    __shared__ int sh_max[T];
     sh_off[threadIdx.x] = s_off;
     sh_ioff[threadIdx.x] = s_ioff;
+    sh_max[threadIdx.x] = mx;
     __syncthreads();
-    // Hillis-Steele inclusive scan over the per-thread sums.
-    for (int d = 1; d < kScanThreads; d <<= 1) {
+    // Hillis-Steele inclusive scan over the per-thread sums (and a max).
+    for (int d = 1; d < T; d <<= 1) {
         int64_t vo = 0, vi = 0;
+        int vm = 0;
         if ((int)threadIdx.x >= d) {
             vo = sh_off[threadIdx.x - d];
             vi = sh_ioff[threadIdx.x - d];
+            vm = sh_max[threadIdx.x - d];
         }
         __syncthreads();
         sh_off[threadIdx.x] += vo;
         sh_ioff[threadIdx.x] += vi;
+        sh_max[threadIdx.x] = max(sh_max[threadIdx.x], vm);
         __syncthreads();
     }
     int64_t run_off = sh_off[threadIdx.x] - s_off;
     int64_t run_ioff = sh_ioff[threadIdx.x] - s_ioff;
     for (int h = h0; h < h1; ++h) {
+        const int n = __ldcg(a.len + h);
         a.off[h] = a.stride > 0 ? (int64_t)h * a.stride : run_off;  // in place: the slab's own dense rows
         a.ioff[h] = run_ioff;
-        run_off += (int64_t)a.len[h] + a.reserve;
-        run_ioff += a.len[h];
+        run_off += (int64_t)n + a.reserve;
+        run_ioff += n;
     }
-    if (threadIdx.x == kScanThreads - 1) {
-        a.off[a.NH] = a.stride > 0 ? (int64_t)a.NH * a.stride : sh_off[kScanThreads - 1];
-        a.ioff[a.NH] = sh_ioff[kScanThreads - 1];
+    if (threadIdx.x == T - 1) {
+        const int64_t total = a.stride > 0 ? (int64_t)a.NH * a.stride : sh_off[T - 1];
+        a.off[a.NH] = total;
+        a.ioff[a.NH] = sh_ioff[T - 1];
+        a.tail[0] = total;
+        a.tail[1] = sh_ioff[T - 1];
+        a.tail[2] = sh_max[T - 1];
     }
+    __syncthreads();  // every ioff is written (this CTA's own global writes)
+    // Kept rows of each layer: NHl = B * Hkv slabs per layer.
+    const int NHl = a.B * a.Hkv;
+    for (int l = threadIdx.x; l < a.L; l += T) a.tail[3 + l] = a.ioff[(l + 1) * NHl] - a.ioff[l * NHl];
 }
 
-__global__ void __launch_bounds__(kMapThreads) write_kernel(const MapArgs a)
+// In-place plans: order[rank(h)] = h, rank = slabs longer than h, or as long
+// with a lower index (a stable sort by length, longest first).
+__global__ void __launch_bounds__(256) order_kernel(const int32_t* __restrict__ len, int NH, int32_t* order)
 {
-    const int h = blockIdx.x, c = blockIdx.y;
-    const SlabView v = slab_view(a, h);
-    const int base = c * kMapChunk;
-    if (base >= v.Tc) return;  // uniform over the CTA
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    __shared__ int warp_cnt[kMapThreads / 32];
-    int64_t out = a.ioff[h] + a.chunk_cnt[(int64_t)h * a.nchunks + c];
-    for (int k = 0; k < kMapIters; ++k) {
-        const int p = base + k * kMapThreads + threadIdx.x;
-        const bool kp = p < v.Tc && keep_pos(v.Urow, p, v.Tc, a.sink, a.recent, a.bin_width);
-        const unsigned bal = __ballot_sync(0xffffffffu, kp);
-        if (lane == 0) warp_cnt[warp] = __popc(bal);
+    __shared__ int tile[1024];
+    const int h = blockIdx.x * blockDim.x + threadIdx.x;
+    const int mine = h < NH ? len[h] : 0;
+    int rank = 0;
+    for (int t0 = 0; t0 < NH; t0 += 1024) {
+        const int n = min(1024, NH - t0);
         __syncthreads();
-        int before = 0, total = 0;
-#pragma unroll
-        for (int w = 0; w < kMapThreads / 32; ++w) {
-            const int n = warp_cnt[w];
-            before += (w < warp) ? n : 0;
-            total += n;
+        for (int i = threadIdx.x; i < n; i += blockDim.x) tile[i] = len[t0 + i];
+        __syncthreads();
+        if (h < NH)
+            for (int i = 0; i < n; ++i) {
+                const int x = tile[i];
+                rank += (x > mine || (x == mine && t0 + i < h)) ? 1 : 0;
+            }
+    }
+    if (h < NH) order[rank] = h;
+}
+
+__global__ void __launch_bounds__(kWriteThreads) write_kernel(const MapArgs a)
+{
+    const int h = blockIdx.x;
+    const int n_h = __ldg(a.len + h);
+    const int r0 = blockIdx.y * kMapChunk;
+    if (r0 >= n_h) return;  // uniform over the CTA
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int2* run = a.runs + (int64_t)h * (a.D + 2);
+    const int nr = __ldg(a.nruns + h);
+    int32_t* dst = a.idx + __ldg(a.ioff + h);
+    // Lane rows: base + 32 k, k < 32 (the warp covers 1024 consecutive rows).
+    const int base = r0 + warp * (kMapChunk / (kWriteThreads / 32)) + lane;
+    if (base >= n_h) return;
+    // Run holding `base`: the last run whose first row is <= base.
+    int lo = 0, hi = nr - 1;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (__ldg(&run[mid].x) <= base)
+            lo = mid;
+        else
+            hi = mid - 1;
+    }
+    int i = lo;
+    int2 cur = __ldg(run + i);
+    int next = i + 1 < nr ? __ldg(&run[i + 1].x) : n_h;
+#pragma unroll 4
+    for (int k = 0; k < 32; ++k) {
+        const int r = base + 32 * k;
+        if (r >= n_h) break;
+        while (r >= next) {
+            ++i;
+            cur = __ldg(run + i);
+            next = i + 1 < nr ? __ldg(&run[i + 1].x) : n_h;
         }
-        if (kp) a.idx[out + before + __popc(bal & ((1u << lane) - 1u))] = p;
-        out += total;
-        __syncthreads();  // warp_cnt is rewritten by the next iteration
+        dst[r] = cur.y + (r - cur.x);
     }
 }
 
@@ -164,21 +225,20 @@ __global__ void __launch_bounds__(kMapThreads) write_kernel(const MapArgs a)
 
 cudaError_t launch_map(const MapArgs& a, cudaStream_t st)
 {
-    const int64_t nu = (int64_t)a.L * a.Hkv * a.D;
-    if (nu > 0) {
-        const int blocks = (int)((nu + 255) / 256 < 4096 ? (nu + 255) / 256 : 4096);
-        union_kernel<<<blocks, 256, 0, st>>>(a.M, a.U, a.L, a.H, a.Hkv, a.D);
-    }
-    dim3 grid(a.NH, a.nchunks);
-    count_kernel<<<grid, kMapThreads, 0, st>>>(a);
-    scan_kernel<<<1, kScanThreads, 0, st>>>(a);
+    if (a.NH < 1) return cudaErrorInvalidValue;
+    const int grid = (a.NH + kRunsThreads / 32 - 1) / (kRunsThreads / 32);
+    runs_kernel<<<grid, kRunsThreads, 0, st>>>(a);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess || !a.order) return e;
+    order_kernel<<<(a.NH + 255) / 256, 256, 0, st>>>(a.len, a.NH, a.order);
     return cudaGetLastError();
 }
 
-cudaError_t launch_map_write(const MapArgs& a, cudaStream_t st)
+cudaError_t launch_map_write(const MapArgs& a, int max_len, cudaStream_t st)
 {
-    dim3 grid(a.NH, a.nchunks);
-    write_kernel<<<grid, kMapThreads, 0, st>>>(a);
+    if (max_len < 1) return cudaSuccess;  // no kept rows: nothing to write
+    dim3 grid(a.NH, (max_len + kMapChunk - 1) / kMapChunk);
+    write_kernel<<<grid, kWriteThreads, 0, st>>>(a);
     return cudaGetLastError();
 }
 

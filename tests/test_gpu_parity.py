@@ -68,6 +68,27 @@ def test_map_edge_lengths(Tc):
     plan.close()
 
 
+def test_map_random_geometries():
+    """Sink or recent window of 0, bins of 1 to 100 positions (runs shorter than
+    a warp's stride), contexts from 0 to the pattern's full span, random
+    patterns and reserves: bit-exact against the oracle's position walk."""
+    rng = np.random.default_rng(17)
+    for trial in range(40):
+        L, Hkv, G, B = int(rng.integers(1, 3)), int(rng.integers(1, 3)), int(rng.integers(1, 5)), int(rng.integers(1, 4))
+        S, R = int(rng.choice([0, 1, 3, 16])), int(rng.choice([0, 1, 5, 33]))
+        W, D = int(rng.choice([1, 2, 7, 31, 32, 33, 100])), int(rng.integers(1, 80))
+        Tc = rng.integers(0, S + R + D * W + 1, size=B).astype(np.int32)
+        if trial % 5 == 0:
+            Tc[:] = S + R + D * W
+        M = (rng.random((L, G * Hkv, D)) < rng.random()).astype(np.uint8)
+        reserve = int(rng.integers(0, 3))
+        sh = dkv.Shape(L=L, H=G * Hkv, H_kv=Hkv, D=D, sink=S, recent=R, bin_width=W)
+        geo = O.Geometry(L=L, H=G * Hkv, Hkv=Hkv, D=D, sink=S, recent=R, bin_width=W)
+        plan = dkv.dkv_map_pattern(M, Tc, sh, reserve_rows=reserve)
+        check_map(plan, O.map_pattern(M, Tc, geo, reserve=reserve))
+        plan.close()
+
+
 @pytest.mark.parametrize("fill", [0, 1])
 def test_map_all_drop_and_all_keep(fill):
     w = wl(T=20000, D=20, W=1000)
