@@ -71,13 +71,6 @@ struct MK {
 #ifndef DKV_MMA_CFG_MULTI
 #define DKV_MMA_CFG_MULTI 2, 12
 #endif
-// Tiles per warp whose rows are prefetched into L2 (after the ring tiles
-// fetched before the wait for the previous kernel), while that kernel drains.
-#ifndef DKV_L2_PREFETCH_TILES
-#define DKV_L2_PREFETCH_TILES 0
-#endif
-constexpr int kL2PrefetchTiles = DKV_L2_PREFETCH_TILES;
-
 template <int G, int NT, bool MULTI>
 using MKFor = typename std::conditional<
     (NT > 1), MK<G, NT, DKV_MMA_CFG_MULTI>,
@@ -438,18 +431,6 @@ __global__ void __launch_bounds__(MKFor<G, NT, MULTI>::NW * 32, 1)
         for (int s = 0; s < PRE && ld.h < hend; ++s) {
             ++inflight;
             cursor_next<TR>(ld, a, tab, hend, wA, wB);
-        }
-        if (kL2PrefetchTiles > 0 && lane == 0) {
-            // The next tiles' K and V rows into L2 while the previous kernel
-            // drains: exactly the segment's rows, all inside the cache.
-            Cursor it = ld;
-            for (int s = 0; s < kL2PrefetchTiles && it.h < hend; ++s) {
-                const int cnt = min(TR, it.s1 - it.x);
-                const int64_t row = it.base + (it.x - it.p0);
-                prefetch_l2_bulk(a.Kc + row * kHeadDim, (uint32_t)cnt * kRowBytes);
-                prefetch_l2_bulk(a.Vc + row * kHeadDim, (uint32_t)cnt * kRowBytes);
-                cursor_next<TR>(it, a, tab, hend, wA, wB);
-            }
         }
         // Everything above reads only the plan, n_appended and the cache rows of
         // earlier steps; q, k_new, v_new, the cache slots written here and the

@@ -79,13 +79,6 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t
         : "memory");
 }
 
-// Bulk prefetch of `bytes` (a multiple of 16) at `src` (16-byte aligned) into
-// L2, with no destination in shared memory and nothing to wait for.
-__device__ __forceinline__ void prefetch_l2_bulk(const void* src, uint32_t bytes)
-{
-    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
-}
-
 __device__ __forceinline__ void fence_proxy_async_smem()
 {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
