@@ -892,12 +892,16 @@ def run_dkv(args, dist):
         with nvtx("pattern export"):
             res["pattern_export"] = time_topk(wl, dev)
         mq = {}
-        for Q in sorted({1, max(1, 8 // wl.G), max(1, 16 // wl.G)}):
+        for Q in sorted({1, max(1, 8 // wl.G), max(1, 16 // wl.G), max(1, 32 // wl.G), max(1, 64 // wl.G)}):
             with nvtx(f"multi-query Q={Q} graph (timed)"):
                 t_q = dist.max(time_multi_query(wl, env, dev, Q, min(steps, 64), warmup))
             rows_q = sum(rows_layer)  # no appends in these calls
+            # K/V rows once for all Q queries, plus every query's q read and out written.
+            bytes_q = step_bytes(wl, rows_q, with_new=False) + (Q - 1) * wl.B * wl.H * wl.head_dim * (2 + 4)
+            gbs_q = bytes_q / t_q / 1e9
             mq[f"Q{Q}"] = {"us_per_step": round(t_q * 1e6, 2), "queries_per_s": round(wl.B * Q * dist.world / t_q, 1),
-                           "gbs": round(step_bytes(wl, rows_q, with_new=False) / t_q / 1e9, 1)}
+                           "columns": Q * wl.G, "kernel": "tcgen05" if Q * wl.G > 16 else "mma.sync",
+                           "gbs": round(gbs_q, 1), "frac_of_hbm": round(gbs_q / peak, 4)}
         res["multi_query"] = mq
     if not args.profile:
         with nvtx("in-place compaction"):

@@ -38,6 +38,7 @@ struct dkv_plan {
     dkv::DecodeConfig cfg_mma{};     // tensor-core kernel of the decode step
     dkv::DecodeConfig cfg_multi1{};  // multi-query, one column tile (tensor-core plans)
     dkv::DecodeConfig cfg_multi{};   // multi-query, two column tiles (tensor-core plans)
+    dkv::DecodeConfig cfg_tc{};      // multi-query, 17 to 64 columns on tcgen05 (tensor-core plans)
     dkv::WorkspaceLayout work{};     // carve-up of d_work
     int cols_cap = 0;                // columns the workspace and counters are sized for
     int use_mma = 0;  // tensor-core decode kernel (needs the cache's row count for its tensor maps)
@@ -169,13 +170,17 @@ dkv_status plan_configs(dkv_plan* p)
         (e = dkv::decode_config_mma(p->G, p->B, 1, &p->cfg_multi1)) != cudaSuccess ||
         (e = dkv::decode_config_mma(p->G, p->B, 2, &p->cfg_multi)) != cudaSuccess)
         return cuda_fail(e, "decode_config (tensor cores)");
-    int64_t ctas = 0, warp_records = 0;
+    if ((e = dkv::decode_config_tc(p->G, p->B, &p->cfg_tc)) != cudaSuccess) return cuda_fail(e, "decode_config (tcgen05)");
+    // Warp records: the mma.sync and fp32 kernels (up to kMaxCols columns); CTA
+    // partials: every kernel, up to kTcMaxCols columns (the tcgen05 kernel).
+    int64_t ctas = p->cfg_tc.nctas, warp_records = 0;
     for (const dkv::DecodeConfig* c : {&p->cfg_f32, &p->cfg_mma, &p->cfg_multi1, &p->cfg_multi}) {
         ctas = std::max<int64_t>(ctas, c->nctas);
         warp_records = std::max<int64_t>(warp_records, (int64_t)c->nctas * c->nwarps);
     }
     p->cols_cap = dkv::kMaxCols;
-    p->work = dkv::workspace_layout(ctas + (int64_t)p->B * p->s.H_kv, warp_records, p->cols_cap);
+    const int64_t NHl = (int64_t)p->B * p->s.H_kv;
+    p->work = dkv::workspace_layout(ctas + NHl, dkv::kTcMaxCols, warp_records, dkv::kMaxCols, NHl);
     return DKV_OK;
 }
 
@@ -601,6 +606,7 @@ dkv_status decode_args(const dkv_plan* p, int32_t layer, const void* q, const vo
     a->work_ml = p->d_work + p->work.work_ml;
     a->warp_o = p->d_work + p->work.warp_o;
     a->warp_ml = p->d_work + p->work.warp_ml;
+    a->tc_bounds = reinterpret_cast<int32_t*>(p->d_work + p->work.bounds);
     if (!aligned16(a->work_o) || !aligned16(a->work_ml) || !aligned16(a->warp_o) || !aligned16(a->warp_ml))
         return fail(DKV_ERR_INVALID_ARG, "split-K workspace regions are not 16-byte aligned");
     a->out = out;
@@ -658,13 +664,23 @@ dkv_status dkv_decode_multi(const dkv_plan* p, int32_t layer, const void* q, int
     dkv::DecodeArgs a;
     dkv_status st = decode_args(p, layer, q, nullptr, nullptr, 0, n_appended, Kc, Vc, scale, out, true, true, &a);
     if (st != DKV_OK) return st;
-    if (num_queries < 1 || num_queries * p->G > dkv::kMaxCols)
+    if (num_queries < 1 || (int64_t)num_queries * p->G > dkv::kTcMaxCols)
         return fail(DKV_ERR_INVALID_ARG, "num_queries=%d: need 1 <= Q and Q*G <= %d (G=%d)", num_queries,
-                    dkv::kMaxCols, p->G);
+                    dkv::kTcMaxCols, p->G);
     if (!p->use_mma)
         return fail(DKV_ERR_INVALID_ARG, "multi-query decode needs the tensor-core kernel (a cache of < 2^31 rows)");
     a.Q = num_queries;
     a.NC = num_queries * p->G;
+    if (a.NC > dkv::kMaxCols) {
+        // More columns than the mma.sync kernels' accumulator registers hold: the
+        // tcgen05 kernel (accumulators in TMEM) and its combine launch.
+        a.nctas = p->cfg_tc.nctas;
+        dkv::CacheMaps maps;
+        const cudaError_t e = dkv::make_cache_maps(a.Kc, a.Vc, p->total_rows, &maps, fault("copy"), 64);
+        if (e != cudaSuccess) return cuda_fail(e, "tensor maps of the packed caches");
+        st = launched(dkv::launch_decode_tc(a, maps, p->cfg_tc, stream), "multi-query decode kernel (tcgen05)");
+        return st == DKV_OK ? ok() : st;
+    }
     // Q = 1 runs the decode step's kernel; more queries the multi-query kernels.
     const dkv::DecodeConfig& cfg = num_queries == 1 ? p->cfg : (a.NC > 8 ? p->cfg_multi : p->cfg_multi1);
     a.nctas = launch_ctas(p, layer, cfg);

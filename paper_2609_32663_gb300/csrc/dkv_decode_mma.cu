@@ -618,8 +618,10 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
 
 }  // namespace
 
-cudaError_t make_cache_maps(const void* Kc, const void* Vc, int64_t rows, CacheMaps* maps, bool short_boxes)
+cudaError_t make_cache_maps(const void* Kc, const void* Vc, int64_t rows, CacheMaps* maps, bool short_boxes,
+                            int box_rows)
 {
+    if (box_rows < 8 || box_rows > 256 || (box_rows & 7)) return cudaErrorInvalidValue;
     if (rows < 1 || rows > kMaxMmaRows) return cudaErrorInvalidValue;
     PFN_cuTensorMapEncodeTiled_v12000 enc = encode_fn();
     if (!enc) return cudaErrorNotSupported;
@@ -627,7 +629,7 @@ cudaError_t make_cache_maps(const void* Kc, const void* Vc, int64_t rows, CacheM
     const cuuint64_t stride[1] = {(cuuint64_t)kRowBytes};
     // short_boxes (fault injection): 8-row boxes deliver half the bytes each
     // stage's mbarrier expects, inside the stage, so every wait runs out.
-    const cuuint32_t box[2] = {64, (cuuint32_t)(short_boxes ? kMmaTR / 2 : kMmaTR)};
+    const cuuint32_t box[2] = {64, (cuuint32_t)(short_boxes ? box_rows / 2 : box_rows)};
     const cuuint32_t elem[2] = {1, 1};
     const void* base[2] = {Kc, Vc};
     CUtensorMap* out[2] = {&maps->k, &maps->v};

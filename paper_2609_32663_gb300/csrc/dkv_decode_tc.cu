@@ -1,0 +1,689 @@
+// Multi-query decode over the packed cache (Sec. 3.4; shared-context reuse,
+// Sec. 4.1) on the fifth-generation tensor cores: tcgen05.mma with operands in
+// shared memory and accumulators in tensor memory (TMEM), for 17 to 64 columns
+// (queries x heads of a KV head's group) per slab.
+//
+// Work split: the layer's rows (every slab end to end, plus the rows appended in
+// earlier steps) are cut into equal contiguous CTA ranges (one CTA per SM), as in
+// the other decode kernels; a CTA walks its range in tiles of 64 rows, slab
+// segment by slab segment. Per tile, one pipeline per CTA:
+//
+//   warp 0 (one lane)   TMA: the tile's K and V rows as four 2-D boxes
+//                       (64 rows x 64 dims, 128-byte swizzle) into a 4-stage ring.
+//   warp 1 (one lane)   MMA: S^T = Q K^T  (M = 128 query-column rows of Q, padded
+//                       with zeros, N = 64 cache rows, K = 128 dims; 8 MMAs) into
+//                       one of two TMEM score buffers, then, one tile behind,
+//                       O^T += V^T P  (M = 128 dims, N = the columns rounded up to
+//                       16, K = 64 rows; V^T read MN-major from the same stage;
+//                       P as a bf16 high part and remainder, two MMAs per k-step)
+//                       into the TMEM output accumulator.
+//   warps 2-5           softmax: thread c owns column c, i.e. TMEM lane c of the
+//                       score buffer (all 64 scores of the tile in its lane): tile
+//                       max, lazily rescaled running max (a column's max moves only
+//                       when a score tops it by kSlack; O is then rescaled in
+//                       TMEM), P = 2^(s - m) written to shared memory as the B
+//                       operand of the next product, V rows past a segment zeroed.
+//                       At a segment's end the same warps read O^T (thread d owns
+//                       dimension d, TMEM lane d) and write the slab's output, or
+//                       the CTA's partial (m, l, o) of each column when the slab
+//                       continues in another CTA.
+//
+// Slabs that span several CTAs are merged by decode_tc_combine_kernel, a separate
+// launch with one CTA per (slab, column): with up to 64 columns a slab's partials
+// are up to 64 x 19 records at the 128K context, too many for the last CTA of
+// the slab to merge alone in time.
+//
+// Every wait is bounded (polls and 2 s); a wait that runs out sets
+// DKV_DEV_TMA_TIMEOUT, the roles stop, the copies and products in flight are
+// drained with the same bound, and TMEM is freed before the CTA exits.
+#include "dkv_decode_common.cuh"
+
+#include <cuda.h>
+
+#include <math.h>
+
+namespace dkv {
+namespace {
+
+constexpr int kTcRows = 64;                    // cache rows per tile
+constexpr int kTcStages = 4;                   // ring stages
+constexpr int kTcBox = kTcRows * 128;          // one TMA box: 64 rows x 64 dims of bf16 (8 KB)
+constexpr int kTcStage = 4 * kTcBox;           // K dims 0-63, K dims 64-127, V dims 0-63, V dims 64-127
+constexpr int kTcThreads = 192;                // warps: 0 TMA, 1 MMA, 2-5 softmax and epilogue
+constexpr int kTcQBytes = 2 * 128 * 128;       // Q as the A operand: 128 rows x 128 dims, two 64-dim halves
+constexpr int kTcPBytes = 2 * kTcMaxCols * 128;  // one P buffer: high and low parts, 64 columns x 64 rows each
+constexpr int kTcTmemCols = 256;               // S buffers at columns 0 and 64, O at 128
+constexpr int kTcSCol = 0, kTcOCol = 128;
+constexpr int kSmBar = 1;                      // named barrier of the softmax warpgroup
+
+// Shared-memory layout, from a 1024-byte aligned base.
+constexpr int kOffRing = 0;
+constexpr int kOffQ = kOffRing + kTcStages * kTcStage;
+constexpr int kOffP = kOffQ + kTcQBytes;
+constexpr int kOffStats = kOffP + 2 * kTcPBytes;           // m[64], l[64], alpha[64] (floats)
+constexpr int kOffFlags = kOffStats + 3 * kTcMaxCols * 4;  // int[16]
+constexpr int kOffBars = kOffFlags + 16 * 4;               // uint64 barriers
+// full[S], empty[S], s_full[2], p_full[2], o_done[2], q_full, fin
+constexpr int kNumBars = 2 * kTcStages + 8;
+constexpr int kOffTmem = kOffBars + kNumBars * 8;
+constexpr int kOffTable = (kOffTmem + 16 + 15) / 16 * 16;
+constexpr int kTcAlign = 1024;
+__host__ __device__ constexpr int tc_smem_bytes(int B) { return kTcAlign + kOffTable + seq_table_bytes(B); }
+static_assert(tc_smem_bytes(kMaxB) <= 227 * 1024, "fits the opt-in shared memory of one CTA");
+
+// Flag slots.
+constexpr int kFlagVote = 0;      // [4] per-warp rescale votes of the softmax warpgroup
+constexpr int kFlagAbort = 4;     // a bounded wait ran out
+constexpr int kFlagOk = 5;        // result of the leader's wait, for the warpgroup
+constexpr int kFlagIssued = 6;    // tiles the TMA lane issued
+constexpr int kFlagConsumed = 7;  // tiles whose copies the MMA lane saw land
+constexpr int kFlagMmaLast = 8;   // the MMA lane issued products (fin must be awaited before freeing TMEM)
+
+// ------------------------------------------------------------ tcgen05 wrappers
+// Shared-memory matrix descriptor: start address, leading and stride byte
+// offsets (16-byte units), descriptor version 1, 128-byte swizzle.
+__device__ __forceinline__ uint64_t sdesc(uint32_t addr, uint32_t lbo, uint32_t sbo)
+{
+    return (uint64_t)((addr >> 4) & 0x3fff) | ((uint64_t)((lbo >> 4) & 0x3fff) << 16) |
+           ((uint64_t)((sbo >> 4) & 0x3fff) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
+// Instruction descriptor of kind::f16: fp32 accumulate, bf16 A and B, the
+// operands' major-ness (0: K-major, 1: MN-major), N and M.
+__device__ __forceinline__ uint32_t idesc(int M, int N, int a_mn, int b_mn)
+{
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)a_mn << 15) | ((uint32_t)b_mn << 16) |
+           ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+__device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t id, uint32_t acc)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a), "l"(b), "r"(id), "r"(acc)
+        : "memory");
+}
+
+// The mbarrier arrives once every product issued so far by this thread is done.
+__device__ __forceinline__ void umma_commit(uint32_t bar)
+{
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+                 : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// 32 consecutive TMEM columns of this thread's lane (warp w reads lanes 32 (w % 4) ..).
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32])
+{
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const float (&v)[32])
+{
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+        "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+        "f"(v[0]), "f"(v[1]), "f"(v[2]), "f"(v[3]), "f"(v[4]), "f"(v[5]), "f"(v[6]), "f"(v[7]), "f"(v[8]),
+        "f"(v[9]), "f"(v[10]), "f"(v[11]), "f"(v[12]), "f"(v[13]), "f"(v[14]), "f"(v[15]), "f"(v[16]),
+        "f"(v[17]), "f"(v[18]), "f"(v[19]), "f"(v[20]), "f"(v[21]), "f"(v[22]), "f"(v[23]), "f"(v[24]),
+        "f"(v[25]), "f"(v[26]), "f"(v[27]), "f"(v[28]), "f"(v[29]), "f"(v[30]), "f"(v[31])
+        : "memory");
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void named_sync(int id, int n) { asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory"); }
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar)
+{
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void tma_box(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar, uint64_t pol)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+        " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
+        "l"(map), "r"(x), "r"(y), "r"(bar), "l"(pol)
+        : "memory");
+}
+
+// Byte offset of 16-byte chunk ch (0..7) of 128-byte row r in a 128-byte-swizzled tile.
+__device__ __forceinline__ int sw128(int r, int ch) { return r * 128 + ((ch ^ (r & 7)) << 4); }
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
+{
+    uint32_t d;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+    return d;
+}
+
+// ------------------------------------------------------------ tiles
+// The CTA's tiles, slab segment by slab segment: a segment is the part of one
+// slab inside the CTA's range [A, B); tiles are 64 rows from the segment's start.
+struct TileWalk {
+    Cursor cu;
+    int hend, A, B;
+    __device__ void begin(const DecodeArgs& a, const SeqTable& t, int hfirst, int hend_, int A_, int B_)
+    {
+        hend = hend_;
+        A = A_;
+        B = B_;
+        cu.h = hfirst;
+        cursor_seek(cu, a, t, hend, A, B);
+    }
+    __device__ bool more() const { return cu.h < hend; }
+    __device__ int cnt() const { return min(kTcRows, cu.s1 - cu.x); }
+    __device__ bool first() const { return cu.x == cu.s0; }
+    __device__ bool last() const { return cu.x + kTcRows >= cu.s1; }
+    __device__ int cache_row() const { return (int)(cu.base + (cu.x - cu.p0)); }
+    __device__ void next(const DecodeArgs& a, const SeqTable& t) { cursor_next<kTcRows>(cu, a, t, hend, A, B); }
+};
+
+// Q of slab h as the A operand: row c (column c: query c / G, head g G + c % G)
+// of 128 bf16 dims, two 64-dim halves, 128-byte swizzle; rows NC.. are zero.
+template <int G>
+__device__ void load_q_tc(const DecodeArgs& a, int h, unsigned char* sQ, int tid)
+{
+    const int b = h / a.Hkv, g = h - b * a.Hkv;
+    for (int i = tid; i < 128 * 16; i += 128) {
+        const int c = i >> 4, ch = i & 15;
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (c < a.NC) {
+            const int qi = c / G, j = c - qi * G;
+            const uint4* src = reinterpret_cast<const uint4*>(a.q + (((int64_t)b * a.Q + qi) * a.H + g * G + j) * kHeadDim);
+            v = __ldg(src + ch);
+        }
+        *reinterpret_cast<uint4*>(sQ + (ch >> 3) * (128 * 128) + sw128(c, ch & 7)) = v;
+    }
+}
+
+// Bounded wait by one lane; true when the phase completed.
+__device__ __forceinline__ bool wait_phase(uint64_t* bar, uint32_t parity) { return mbar_wait(smem_u32(bar), parity); }
+
+template <int G>
+__global__ void __launch_bounds__(kTcThreads, 1)
+    decode_tc_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ CacheMaps maps)
+{
+    extern __shared__ __align__(128) unsigned char smem_raw[];
+    unsigned char* sm = smem_raw + ((kTcAlign - (smem_u32(smem_raw) & (kTcAlign - 1))) & (kTcAlign - 1));
+    unsigned char* ring = sm + kOffRing;
+    unsigned char* sQ = sm + kOffQ;
+    unsigned char* sP = sm + kOffP;
+    float* st_m = reinterpret_cast<float*>(sm + kOffStats);
+    float* st_l = st_m + kTcMaxCols;
+    float* st_a = st_l + kTcMaxCols;
+    volatile int* flags = reinterpret_cast<volatile int*>(sm + kOffFlags);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sm + kOffBars);
+    uint64_t* full = bars;
+    uint64_t* empty = bars + kTcStages;
+    uint64_t* s_full = bars + 2 * kTcStages;
+    uint64_t* p_full = s_full + 2;
+    uint64_t* o_done = p_full + 2;
+    uint64_t* q_full = o_done + 2;
+    uint64_t* fin = q_full + 1;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + kOffTmem);
+    const SeqTable tab = seq_table_at(sm + kOffTable, a);
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int NHl = a.B * a.Hkv;
+    const int c = blockIdx.x;
+
+    if (warp == 0)
+        build_seq_table(a, tab, false);
+    else
+        load_slab_cache(a, tab, 32, kTcThreads - 32);
+    if (tid == 32) {
+        for (int i = 0; i < 2 * kTcStages + 6; ++i) mbar_init(smem_u32(&bars[i]), 1);
+        mbar_init(smem_u32(q_full), 1);
+        mbar_init(smem_u32(fin), 1);
+        for (int i = 0; i < 16; ++i) flags[i] = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        fence_proxy_async_smem();
+    }
+    __syncthreads();
+    pdl_launch_dependents();
+
+    const int R = slab_start(a, tab, NHl);
+    if (c == 0 && warp == 2) {
+        // Slab bounds for the combine launch (after the wait: the previous kernel may read them).
+        pdl_wait();
+        for (int h = lane; h <= NHl; h += 32) a.tc_bounds[h] = slab_start(a, tab, h);
+    }
+    const int A = part_start(c, R, a.nctas), Bc = part_start(c + 1, R, a.nctas);
+    if (A >= Bc) return;  // uniform: this CTA has no rows (no TMEM taken yet)
+    const int hfirst = slab_containing(a, tab, NHl, A);
+    const int hend = slab_containing(a, tab, NHl, Bc - 1) + 1;
+
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                     "r"(kTcTmemCols));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    const int NC = a.NC;
+    const int NCpad = (NC + 15) & ~15;
+    const float cs = a.qscale;
+
+    if (warp == 0) {
+        // ---------------------------------------------------------------- TMA
+        if (lane == 0) {
+            const uint64_t pol = evict_first_policy();
+            TileWalk w;
+            w.begin(a, tab, hfirst, hend, A, Bc);
+            int t = 0;
+            for (; w.more(); ++t, w.next(a, tab)) {
+                if (flags[kFlagAbort]) break;
+                const int s = t % kTcStages;
+                if (t >= kTcStages && !wait_phase(&empty[s], ((t / kTcStages) - 1) & 1)) {
+                    atomicOr(a.status, 0x2 /* DKV_DEV_TMA_TIMEOUT */);
+                    flags[kFlagAbort] = 1;
+                    break;
+                }
+                if (t == PRE) pdl_wait();  // later copies after the previous kernel, as in the other kernels
+                const int row = w.cache_row();
+                const uint32_t bar = smem_u32(&full[s]);
+                const uint32_t dst = smem_u32(ring + s * kTcStage);
+                mbar_arrive_expect_tx(bar, kTcStage);
+                tma_box(dst, &maps.k, 0, row, bar, pol);
+                tma_box(dst + kTcBox, &maps.k, 64, row, bar, pol);
+                tma_box(dst + 2 * kTcBox, &maps.v, 0, row, bar, pol);
+                tma_box(dst + 3 * kTcBox, &maps.v, 64, row, bar, pol);
+            }
+            flags[kFlagIssued] = t;
+        }
+    } else if (warp == 1) {
+        // ---------------------------------------------------------------- MMA
+        if (lane == 0) {
+            const uint32_t id1 = idesc(128, kTcRows, 0, 0);
+            const uint32_t id2 = idesc(128, NCpad, 1, 0);
+            TileWalk w;
+            w.begin(a, tab, hfirst, hend, A, Bc);
+            int t = 0, seg = 0;
+            bool prev_first = false, issued = false, ok = true;
+            // O^T += V^T P for tile u (its stage's V, its P buffer), then release the stage.
+            auto mma2 = [&](int u, bool first_of_seg) -> bool {
+                const int b = u & 1, s = u % kTcStages;
+                if (!wait_phase(&p_full[b], (u >> 1) & 1)) return false;
+                tc_fence_after();
+                const uint32_t v0 = smem_u32(ring + s * kTcStage + 2 * kTcBox);
+                const uint32_t p0 = smem_u32(sP + b * kTcPBytes);
+#pragma unroll
+                for (int k = 0; k < kTcRows / 16; ++k) {
+                    const uint64_t av = sdesc(v0 + k * 2048, kTcBox, 1024);
+                    umma(tmem + kTcOCol, av, sdesc(p0 + k * 32, 16, 1024), id2, (first_of_seg && k == 0) ? 0u : 1u);
+                    umma(tmem + kTcOCol, av, sdesc(p0 + kTcMaxCols * 128 + k * 32, 16, 1024), id2, 1u);
+                }
+                umma_commit(smem_u32(&o_done[b]));
+                umma_commit(smem_u32(&empty[s]));
+                return true;
+            };
+            for (; w.more(); ++t, w.next(a, tab)) {
+                if (flags[kFlagAbort]) {
+                    ok = false;
+                    break;
+                }
+                const int s = t % kTcStages, b = t & 1;
+                const bool first = w.first();
+                if (!wait_phase(&full[s], (t / kTcStages) & 1)) {
+                    ok = false;
+                    break;
+                }
+                flags[kFlagConsumed] = t + 1;
+                if (first && !wait_phase(q_full, seg++ & 1)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                // S^T[128 x 64] = Q[128 x 128] K^T: k-steps of 16 dims (+32 B inside a 64-dim half).
+                const uint32_t q0 = smem_u32(sQ), k0 = smem_u32(ring + s * kTcStage);
+#pragma unroll
+                for (int k = 0; k < 8; ++k)
+                    umma(tmem + kTcSCol + b * kTcRows, sdesc(q0 + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024),
+                         sdesc(k0 + (k >> 2) * kTcBox + (k & 3) * 32, 16, 1024), id1, k > 0 ? 1u : 0u);
+                umma_commit(smem_u32(&s_full[b]));
+                issued = true;
+                if (t > 0 && !mma2(t - 1, prev_first)) {
+                    ok = false;
+                    break;
+                }
+                prev_first = first;
+            }
+            if (ok && t > 0 && !mma2(t - 1, prev_first)) ok = false;
+            if (!ok) {
+                atomicOr(a.status, 0x2 /* DKV_DEV_TMA_TIMEOUT */);
+                flags[kFlagAbort] = 1;
+            }
+            flags[kFlagMmaLast] = issued ? 1 : 0;
+        }
+    } else {
+        // ---------------------------------------------------------------- softmax and epilogue
+        const int L = 32 * (warp & 3) + lane;       // this thread's TMEM lane: column L of S, dimension L of O
+        const int wg = tid - 64;                    // 0..127 within the warpgroup
+        const bool leader = wg == 0;
+        const uint32_t lane_addr = (uint32_t)(32 * (warp & 3)) << 16;
+        pdl_wait();  // q and the outputs belong to the previous kernel's epoch
+        TileWalk w;
+        w.begin(a, tab, hfirst, hend, A, Bc);
+        load_q_tc<G>(a, w.cu.h, sQ, wg);
+        fence_proxy_async_smem();
+        named_sync(kSmBar, 128);
+        if (leader) mbar_arrive(smem_u32(q_full));
+        float m = -INFINITY, l = 0.f;
+        int t = 0;
+        for (; w.more(); ++t, w.next(a, tab)) {
+            const int b = t & 1, s = t % kTcStages;
+            const int cnt = w.cnt();
+            const bool first = w.first(), last = w.last();
+            // The tile's scores, and the end of the product that last read P buffer b.
+            if (leader) {
+                bool ok = !flags[kFlagAbort] && wait_phase(&s_full[b], (t >> 1) & 1);
+                if (ok && t >= 2) ok = wait_phase(&o_done[b], ((t - 2) >> 1) & 1);
+                if (!ok) {
+                    atomicOr(a.status, 0x2 /* DKV_DEV_TMA_TIMEOUT */);
+                    flags[kFlagAbort] = 1;
+                }
+                flags[kFlagOk] = ok;
+                tc_fence_before();
+            }
+            named_sync(kSmBar, 128);
+            if (!flags[kFlagOk]) break;
+            tc_fence_after();
+            float sc[kTcRows];
+            {
+                float v[32];
+                tmem_ld32(tmem + lane_addr + kTcSCol + b * kTcRows, v);
+#pragma unroll
+                for (int i = 0; i < 32; ++i) sc[i] = v[i];
+                tmem_ld32(tmem + lane_addr + kTcSCol + b * kTcRows + 32, v);
+#pragma unroll
+                for (int i = 0; i < 32; ++i) sc[32 + i] = v[i];
+            }
+            const bool live = L < NC;
+            float mt = -INFINITY;
+#pragma unroll
+            for (int r = 0; r < kTcRows; ++r) {
+                sc[r] = (r < cnt) ? sc[r] * cs : -INFINITY;
+                mt = fmaxf(mt, sc[r]);
+            }
+            if (!live) mt = -INFINITY;
+            if (first) {
+                m = mt;
+                l = 0.f;
+            } else {
+                // Lazy rescale: only when a column's tile max tops its running max by kSlack.
+                const bool vote = live && mt > m + kSlack;
+                const unsigned any = __ballot_sync(kFull, vote);
+                if (lane == 0) flags[kFlagVote + (warp & 3)] = any != 0;
+                named_sync(kSmBar, 128);
+                const bool rescale = flags[kFlagVote] | flags[kFlagVote + 1] | flags[kFlagVote + 2] | flags[kFlagVote + 3];
+                if (rescale) {
+                    float alpha = 1.f;
+                    if (vote) {
+                        alpha = ex2(m - mt);
+                        m = mt;
+                        l *= alpha;
+                    }
+                    if (L < kTcMaxCols) st_a[L] = alpha;
+                    // O^T of every dimension, column by column, once the product of tile t-1 is done.
+                    if (leader) {
+                        const bool ok = wait_phase(&o_done[b ^ 1], ((t - 1) >> 1) & 1);
+                        if (!ok) {
+                            atomicOr(a.status, 0x2 /* DKV_DEV_TMA_TIMEOUT */);
+                            flags[kFlagAbort] = 1;
+                        }
+                        flags[kFlagOk] = ok;
+                        tc_fence_before();
+                    }
+                    named_sync(kSmBar, 128);
+                    if (!flags[kFlagOk]) break;
+                    tc_fence_after();
+                    for (int c0 = 0; c0 < NCpad; c0 += 32) {
+                        float v[32];
+                        tmem_ld32(tmem + lane_addr + kTcOCol + c0, v);
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) v[i] *= (c0 + i < NC) ? st_a[c0 + i] : 1.f;
+                        tmem_st32(tmem + lane_addr + kTcOCol + c0, v);
+                    }
+                }
+            }
+            // P = 2^(s - m) as bf16 high part and remainder: row L (column L) of the B operand.
+            if (L < NCpad) {
+                const float ref = (m == -INFINITY) ? 0.f : m;
+                unsigned char* ph = sP + b * kTcPBytes + L * 128;
+                unsigned char* pl = ph + kTcMaxCols * 128;
+#pragma unroll
+                for (int ch = 0; ch < 8; ++ch) {
+                    uint32_t hi[4], lo[4];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const float p0 = live ? ex2(sc[8 * ch + 2 * i] - ref) : 0.f;  // 2^-inf = 0 past the segment
+                        const float p1 = live ? ex2(sc[8 * ch + 2 * i + 1] - ref) : 0.f;
+                        l += p0 + p1;
+                        hi[i] = pack_bf16(p0, p1);
+                        lo[i] = pack_bf16(p0 - __uint_as_float(hi[i] << 16), p1 - __uint_as_float(hi[i] & 0xffff0000u));
+                    }
+                    const int off = (ch ^ (L & 7)) << 4;
+                    *reinterpret_cast<uint4*>(ph + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+                    *reinterpret_cast<uint4*>(pl + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+                }
+            }
+            if (cnt < kTcRows) {
+                // V rows past the segment: zeros (their p is 0, but 0 * inf or 0 * nan would not be).
+                unsigned char* v0 = ring + s * kTcStage + 2 * kTcBox;
+                for (int i = wg; i < (kTcRows - cnt) * 16; i += 128) {
+                    const int r = cnt + (i >> 4), k = i & 15;
+                    *reinterpret_cast<uint4*>(v0 + (k >> 3) * kTcBox + r * 128 + ((k & 7) << 4)) =
+                        make_uint4(0u, 0u, 0u, 0u);
+                }
+            }
+            fence_proxy_async_smem();
+            tc_fence_before();
+            named_sync(kSmBar, 128);
+            if (leader) mbar_arrive(smem_u32(&p_full[b]));
+            if (!last) continue;
+
+            // ---- end of a segment: the next segment's Q, then this one's output or partial.
+            const int h = w.cu.h, p0h = w.cu.p0, p1h = w.cu.p0 + w.cu.n_h;
+            const bool whole = w.cu.s0 == p0h && w.cu.s1 == p1h;
+            bool has_next = false;
+            {
+                TileWalk nx = w;
+                nx.next(a, tab);
+                has_next = nx.more();
+                if (has_next) {
+                    load_q_tc<G>(a, nx.cu.h, sQ, wg);
+                    fence_proxy_async_smem();
+                }
+            }
+            if (L < NC) {
+                st_m[L] = m;
+                st_l[L] = l;
+            }
+            named_sync(kSmBar, 128);
+            // The next segment's Q is in place: its first S product may start. (It must be
+            // released before the wait below: the MMA lane issues this tile's O product
+            // only after that S product.)
+            if (leader && has_next) mbar_arrive(smem_u32(q_full));
+            if (leader) {
+                const bool ok = wait_phase(&o_done[b], (t >> 1) & 1);
+                if (!ok) {
+                    atomicOr(a.status, 0x2 /* DKV_DEV_TMA_TIMEOUT */);
+                    flags[kFlagAbort] = 1;
+                }
+                flags[kFlagOk] = ok;
+                tc_fence_before();
+            }
+            named_sync(kSmBar, 128);
+            if (!flags[kFlagOk]) break;
+            tc_fence_after();
+            const int bq = h / a.Hkv, g = h - bq * a.Hkv;
+            const int64_t slot = (int64_t)c + h;
+            for (int c0 = 0; c0 < NCpad; c0 += 32) {
+                float v[32];
+                tmem_ld32(tmem + lane_addr + kTcOCol + c0, v);
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    const int cc = c0 + i;
+                    if (cc >= NC) break;
+                    if (whole) {
+                        const float lc = st_l[cc];
+                        a.out[out_row<G>(a, bq, g, cc) * kHeadDim + L] = lc > 0.f ? v[i] / lc : 0.f;
+                    } else {
+                        a.work_o[(slot * NC + cc) * kHeadDim + L] = v[i];
+                    }
+                }
+            }
+            if (!whole && L < NC)
+                *reinterpret_cast<float2*>(a.work_ml + (slot * NC + L) * 2) = make_float2(m, l);
+            m = -INFINITY;
+            l = 0.f;
+            // st_m / st_l are rewritten at the next segment's end, after this one's reads.
+            named_sync(kSmBar, 128);
+        }
+    }
+
+    // ---------------------------------------------------------------- teardown
+    tc_fence_before();
+    __syncthreads();
+    if (flags[kFlagAbort]) {
+        // Drain what is still in flight, with the same bound, before the CTA exits.
+        if (tid == 0) {
+            const int issued = flags[kFlagIssued], consumed = flags[kFlagConsumed];
+            for (int u = max(consumed, issued - kTcStages); u < issued; ++u)
+                wait_phase(&full[u % kTcStages], (u / kTcStages) & 1);
+        }
+        if (tid == 32 && flags[kFlagMmaLast]) {
+            umma_commit(smem_u32(fin));
+            wait_phase(fin, 0);
+        }
+        tc_fence_before();
+        __syncthreads();
+    }
+    tc_fence_after();
+    if (warp == 1)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTcTmemCols));
+}
+
+// Merge of the CTA partials of slab h, column j (one CTA of 128 threads, thread d
+// = dimension d): slabs wholly inside one CTA were written by the decode kernel;
+// slabs with no rows get zeros.
+template <int G>
+__global__ void __launch_bounds__(128) decode_tc_combine_kernel(const DecodeArgs a)
+{
+    pdl_launch_dependents();
+    pdl_wait();
+    const int NC = a.NC;
+    const int h = blockIdx.x / NC, j = blockIdx.x - h * NC;
+    const int NHl = a.B * a.Hkv;
+    const int R = a.tc_bounds[NHl];
+    const int p0 = a.tc_bounds[h], p1 = a.tc_bounds[h + 1];
+    const int b = h / a.Hkv, g = h - b * a.Hkv;
+    float* dst = a.out + out_row<G>(a, b, g, j) * kHeadDim;
+    const int d = threadIdx.x;
+    if (p1 <= p0) {
+        dst[d] = 0.f;
+        return;
+    }
+    const int P = a.nctas;
+    int c0 = 0, c1 = 0;
+    const int nct = ctas_of_slab(p0, p1, R, P, &c0, &c1);
+    if (nct <= 1) return;
+    const bool all_live = R >= P;
+    float M = -INFINITY;
+    for (int cc = c0; cc <= c1; ++cc)
+        if (all_live || part_start(cc, R, P) < part_start(cc + 1, R, P))
+            M = fmaxf(M, __ldcg(a.work_ml + (((int64_t)cc + h) * NC + j) * 2));
+    float O = 0.f, Ls = 0.f;
+#pragma unroll 4
+    for (int cc = c0; cc <= c1; ++cc) {
+        if (!(all_live || part_start(cc, R, P) < part_start(cc + 1, R, P))) continue;
+        const int64_t sj = ((int64_t)cc + h) * NC + j;
+        const float2 ml = __ldcg(reinterpret_cast<const float2*>(a.work_ml + sj * 2));
+        const float f = (ml.x == -INFINITY) ? 0.f : ex2(ml.x - M);
+        Ls = fmaf(ml.y, f, Ls);
+        O = fmaf(__ldcg(a.work_o + sj * kHeadDim + d), f, O);
+    }
+    dst[d] = Ls > 0.f ? O / Ls : 0.f;
+}
+
+template <int G>
+cudaError_t config_tc_g(int B, DecodeConfig* cfg)
+{
+    const int smem = tc_smem_bytes(B);
+    cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    int dev = 0, sms = 0, per_sm = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+    if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_tc_kernel<G>, kTcThreads, smem)) !=
+        cudaSuccess)
+        return e;
+    if (per_sm < 1) return cudaErrorInvalidConfiguration;
+    cfg->nctas = sms;  // one CTA per SM: the TMEM allocation never waits for another CTA's
+    cfg->nwarps = kTcThreads / 32;
+    cfg->smem_bytes = smem;
+    return cudaSuccess;
+}
+
+template <int G>
+cudaError_t launch_tc_g(const DecodeArgs& a, const CacheMaps& maps, const DecodeConfig& cfg, cudaStream_t st)
+{
+    if (cfg.nwarps != kTcThreads / 32 || cfg.smem_bytes < tc_smem_bytes(a.B) || a.nctas < 1 || a.nctas > cfg.nctas ||
+        a.NC < 1 || a.NC > kTcMaxCols || !a.tc_bounds)
+        return cudaErrorInvalidConfiguration;
+    cudaError_t e = launch_pdl(decode_tc_kernel<G>, a.nctas, kTcThreads, cfg.smem_bytes, st, a, maps);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(decode_tc_combine_kernel<G>, a.B * a.Hkv * a.NC, 128, 0, st, a);
+}
+
+}  // namespace
+
+cudaError_t decode_config_tc(int G, int B, DecodeConfig* cfg)
+{
+    if (B < 1 || B > kMaxB) return cudaErrorInvalidValue;
+    switch (G) {
+        case 1: return config_tc_g<1>(B, cfg);
+        case 2: return config_tc_g<2>(B, cfg);
+        case 3: return config_tc_g<3>(B, cfg);
+        case 4: return config_tc_g<4>(B, cfg);
+        case 5: return config_tc_g<5>(B, cfg);
+        case 6: return config_tc_g<6>(B, cfg);
+        case 7: return config_tc_g<7>(B, cfg);
+        case 8: return config_tc_g<8>(B, cfg);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+cudaError_t launch_decode_tc(const DecodeArgs& a, const CacheMaps& maps, const DecodeConfig& cfg, cudaStream_t st)
+{
+    switch (a.G) {
+        case 1: return launch_tc_g<1>(a, maps, cfg, st);
+        case 2: return launch_tc_g<2>(a, maps, cfg, st);
+        case 3: return launch_tc_g<3>(a, maps, cfg, st);
+        case 4: return launch_tc_g<4>(a, maps, cfg, st);
+        case 5: return launch_tc_g<5>(a, maps, cfg, st);
+        case 6: return launch_tc_g<6>(a, maps, cfg, st);
+        case 7: return launch_tc_g<7>(a, maps, cfg, st);
+        case 8: return launch_tc_g<8>(a, maps, cfg, st);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+}  // namespace dkv
