@@ -391,7 +391,7 @@ def time_multi_query(wl, env, dev, Q, steps, warmup):
     return e0.elapsed_time(e1) * 1e-3 / steps
 
 
-def profile_multi_query(wl, env, dev, Qs=(2, 4)):
+def profile_multi_query(wl, env, dev, Qs=(2, 4, 8, 16)):
     """Eager dkv_decode_multi launches, one per layer for each Q, untimed: the
     timed multi-query runs are graph replays, and these are the launches a
     profiler selects."""
@@ -399,7 +399,7 @@ def profile_multi_query(wl, env, dev, Qs=(2, 4)):
 
     import paper_2609_32663_gb300.dkv as dkv
     n_app = torch.zeros(wl.B, dtype=torch.int32, device=dev)
-    for Q in Qs:
+    for Q in (q for q in Qs if q * wl.G <= 64):
         q = torch.randn((wl.B, Q, wl.H, wl.head_dim), device=dev).to(torch.bfloat16)
         out = torch.empty((wl.B, Q, wl.H, wl.head_dim), dtype=torch.float32, device=dev)
         for layer in range(wl.L):
