@@ -10,23 +10,26 @@
 //
 //   warp 0 (one lane)   TMA: the tile's K and V rows as four 2-D boxes
 //                       (64 rows x 64 dims, 128-byte swizzle) into a 4-stage ring.
-//   warp 1 (one lane)   MMA: S^T = Q K^T  (M = 128 query-column rows of Q, padded
-//                       with zeros, N = 64 cache rows, K = 128 dims; 8 MMAs) into
-//                       one of two TMEM score buffers, then, one tile behind,
-//                       O^T += V^T P  (M = 128 dims, N = the columns rounded up to
-//                       16, K = 64 rows; V^T read MN-major from the same stage;
-//                       P as a bf16 high part and remainder, two MMAs per k-step)
-//                       into the TMEM output accumulator.
-//   warps 2-5           softmax: thread c owns column c, i.e. TMEM lane c of the
-//                       score buffer (all 64 scores of the tile in its lane): tile
-//                       max, lazily rescaled running max (a column's max moves only
-//                       when a score tops it by kSlack; O is then rescaled in
-//                       TMEM), P = 2^(s - m) written to shared memory as the B
-//                       operand of the next product, V rows past a segment zeroed.
-//                       At a segment's end the same warps read O^T (thread d owns
-//                       dimension d, TMEM lane d) and write the slab's output, or
-//                       the CTA's partial (m, l, o) of each column when the slab
-//                       continues in another CTA.
+//   warp 1 (one lane)   MMA: S^T = Q K^T  (M = 64 query-column rows of Q, zero
+//                       past the last column, N = 64 cache rows, K = 128 dims;
+//                       8 MMAs) into one of two TMEM score buffers, then, one tile
+//                       behind, O^T += V^T P  (M = 128 dims, N = the columns
+//                       rounded up to 16, K = 64 rows; V^T read MN-major from the
+//                       same stage; P as a bf16 high part and remainder, two MMAs
+//                       per k-step) into the TMEM output accumulator.
+//   warps 2-9           softmax: with M = 64, row c of S^T (column c) sits in
+//                       TMEM lane 32 (c / 16) + c % 16. Warps 2-5 take rows 0-31
+//                       of the tile and warps 6-9 rows 32-63, one column a thread
+//                       (lanes 0-15 of each warp): half-tile max, exchanged once
+//                       per tile, lazily rescaled running max (a column's max
+//                       moves only when a score tops it by kSlack; O is then
+//                       rescaled in TMEM), P = 2^(s - m) written to shared memory
+//                       as the B operand of the next product, V rows past a
+//                       segment zeroed. At a segment's end the same warps read
+//                       O^T (thread d of a warp quarter owns dimension d, TMEM lane
+//                       d; the two halves take 32 columns each) and write the
+//                       slab's output, or the CTA's partial (m, l, o) of each
+//                       column when the slab continues in another CTA.
 //
 // Slabs that span several CTAs are merged by decode_tc_combine_kernel, a separate
 // launch with one CTA per (slab, column): with up to 64 columns a slab's partials
@@ -49,19 +52,22 @@ constexpr int kTcRows = 64;                    // cache rows per tile
 constexpr int kTcStages = 4;                   // ring stages
 constexpr int kTcBox = kTcRows * 128;          // one TMA box: 64 rows x 64 dims of bf16 (8 KB)
 constexpr int kTcStage = 4 * kTcBox;           // K dims 0-63, K dims 64-127, V dims 0-63, V dims 64-127
-constexpr int kTcThreads = 192;                // warps: 0 TMA, 1 MMA, 2-5 softmax and epilogue
-constexpr int kTcQBytes = 2 * 128 * 128;       // Q as the A operand: 128 rows x 128 dims, two 64-dim halves
+constexpr int kTcThreads = 320;                // warps: 0 TMA, 1 MMA, 2-9 softmax and epilogue
+constexpr int kTcSoft = 256;                   // threads of the softmax warps
+constexpr int kTcQRows = 64;                   // M of the score product: the most columns
+constexpr int kTcQHalf = kTcQRows * 128;       // one 64-dim half of Q (8 KB)
+constexpr int kTcQBytes = 2 * kTcQHalf;        // Q as the A operand: 64 rows x 128 dims
 constexpr int kTcPBytes = 2 * kTcMaxCols * 128;  // one P buffer: high and low parts, 64 columns x 64 rows each
 constexpr int kTcTmemCols = 256;               // S buffers at columns 0 and 64, O at 128
 constexpr int kTcSCol = 0, kTcOCol = 128;
-constexpr int kSmBar = 1;                      // named barrier of the softmax warpgroup
+constexpr int kSmBar = 1;                      // named barrier of the softmax warps
 
 // Shared-memory layout, from a 1024-byte aligned base.
 constexpr int kOffRing = 0;
 constexpr int kOffQ = kOffRing + kTcStages * kTcStage;
 constexpr int kOffP = kOffQ + kTcQBytes;
-constexpr int kOffStats = kOffP + 2 * kTcPBytes;           // m[64], l[64], alpha[64] (floats)
-constexpr int kOffFlags = kOffStats + 3 * kTcMaxCols * 4;  // int[16]
+constexpr int kOffStats = kOffP + 2 * kTcPBytes;           // half maxima [2][64], half sums [2][64], alpha[64] (floats)
+constexpr int kOffFlags = kOffStats + 5 * kTcMaxCols * 4;  // int[16]
 constexpr int kOffBars = kOffFlags + 16 * 4;               // uint64 barriers
 // full[S], empty[S], s_full[2], p_full[2], o_done[2], q_full, fin
 constexpr int kNumBars = 2 * kTcStages + 8;
@@ -72,12 +78,12 @@ __host__ __device__ constexpr int tc_smem_bytes(int B) { return kTcAlign + kOffT
 static_assert(tc_smem_bytes(kMaxB) <= 227 * 1024, "fits the opt-in shared memory of one CTA");
 
 // Flag slots.
-constexpr int kFlagVote = 0;      // [4] per-warp rescale votes of the softmax warpgroup
-constexpr int kFlagAbort = 4;     // a bounded wait ran out
-constexpr int kFlagOk = 5;        // result of the leader's wait, for the warpgroup
-constexpr int kFlagIssued = 6;    // tiles the TMA lane issued
-constexpr int kFlagConsumed = 7;  // tiles whose copies the MMA lane saw land
-constexpr int kFlagMmaLast = 8;   // the MMA lane issued products (fin must be awaited before freeing TMEM)
+constexpr int kFlagVote = 0;      // [8] per-warp rescale votes of the softmax warps
+constexpr int kFlagAbort = 8;     // a bounded wait ran out
+constexpr int kFlagOk = 9;        // result of the leader's wait, for the softmax warps
+constexpr int kFlagIssued = 10;   // tiles the TMA lane issued
+constexpr int kFlagConsumed = 11;  // tiles whose copies the MMA lane saw land
+constexpr int kFlagMmaLast = 12;  // the MMA lane issued products (fin must be awaited before freeing TMEM)
 
 // ------------------------------------------------------------ tcgen05 wrappers
 // Shared-memory matrix descriptor: start address, leading and stride byte
@@ -199,7 +205,7 @@ template <int G>
 __device__ void load_q_tc(const DecodeArgs& a, int h, unsigned char* sQ, int tid)
 {
     const int b = h / a.Hkv, g = h - b * a.Hkv;
-    for (int i = tid; i < 128 * 16; i += 128) {
+    for (int i = tid; i < kTcQRows * 16; i += kTcSoft) {
         const int c = i >> 4, ch = i & 15;
         uint4 v = make_uint4(0u, 0u, 0u, 0u);
         if (c < a.NC) {
@@ -207,7 +213,7 @@ __device__ void load_q_tc(const DecodeArgs& a, int h, unsigned char* sQ, int tid
             const uint4* src = reinterpret_cast<const uint4*>(a.q + (((int64_t)b * a.Q + qi) * a.H + g * G + j) * kHeadDim);
             v = __ldg(src + ch);
         }
-        *reinterpret_cast<uint4*>(sQ + (ch >> 3) * (128 * 128) + sw128(c, ch & 7)) = v;
+        *reinterpret_cast<uint4*>(sQ + (ch >> 3) * kTcQHalf + sw128(c, ch & 7)) = v;
     }
 }
 
@@ -224,8 +230,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     unsigned char* sQ = sm + kOffQ;
     unsigned char* sP = sm + kOffP;
     float* st_m = reinterpret_cast<float*>(sm + kOffStats);
-    float* st_l = st_m + kTcMaxCols;
-    float* st_a = st_l + kTcMaxCols;
     volatile int* flags = reinterpret_cast<volatile int*>(sm + kOffFlags);
     uint64_t* bars = reinterpret_cast<uint64_t*>(sm + kOffBars);
     uint64_t* full = bars;
@@ -311,7 +315,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     } else if (warp == 1) {
         // ---------------------------------------------------------------- MMA
         if (lane == 0) {
-            const uint32_t id1 = idesc(128, kTcRows, 0, 0);
+            const uint32_t id1 = idesc(kTcQRows, kTcRows, 0, 0);
             const uint32_t id2 = idesc(128, NCpad, 1, 0);
             TileWalk w;
             w.begin(a, tab, hfirst, hend, A, Bc);
@@ -351,11 +355,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     break;
                 }
                 tc_fence_after();
-                // S^T[128 x 64] = Q[128 x 128] K^T: k-steps of 16 dims (+32 B inside a 64-dim half).
+                // S^T[64 x 64] = Q[64 x 128] K^T: k-steps of 16 dims (+32 B inside a 64-dim half).
                 const uint32_t q0 = smem_u32(sQ), k0 = smem_u32(ring + s * kTcStage);
 #pragma unroll
                 for (int k = 0; k < 8; ++k)
-                    umma(tmem + kTcSCol + b * kTcRows, sdesc(q0 + (k >> 2) * (128 * 128) + (k & 3) * 32, 16, 1024),
+                    umma(tmem + kTcSCol + b * kTcRows, sdesc(q0 + (k >> 2) * kTcQHalf + (k & 3) * 32, 16, 1024),
                          sdesc(k0 + (k >> 2) * kTcBox + (k & 3) * 32, 16, 1024), id1, k > 0 ? 1u : 0u);
                 umma_commit(smem_u32(&s_full[b]));
                 issued = true;
@@ -374,18 +378,29 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         }
     } else {
         // ---------------------------------------------------------------- softmax and epilogue
-        const int L = 32 * (warp & 3) + lane;       // this thread's TMEM lane: column L of S, dimension L of O
-        const int wg = tid - 64;                    // 0..127 within the warpgroup
+        const int sw = warp - 2;                    // 0..7
+        const int grp = sw >> 2;                    // row half of the tile (scores), column chunk (O)
+        const int quarter = warp & 3;               // TMEM lane quarter this warp may access
+        const int wg = tid - 64;                    // 0..255 within the softmax warps
         const bool leader = wg == 0;
-        const uint32_t lane_addr = (uint32_t)(32 * (warp & 3)) << 16;
+        const uint32_t lane_addr = (uint32_t)(32 * quarter) << 16;
+        // Scores: column c = 16 quarter + lane (lanes 0-15), rows 32 grp .. 32 grp + 31.
+        const int col = 16 * quarter + lane;
+        const bool live = lane < 16 && col < NC;
+        float* half_max = st_m;                     // [2][64]
+        float* half_sum = st_m + 2 * kTcMaxCols;    // [2][64]
+        float* st_alpha = st_m + 4 * kTcMaxCols;    // [64]
+        // O: dimension d = 32 quarter + lane, columns 32 grp .. 32 grp + 31.
+        const int dim = 32 * quarter + lane;
+        const int oc0 = 32 * grp;
         pdl_wait();  // q and the outputs belong to the previous kernel's epoch
         TileWalk w;
         w.begin(a, tab, hfirst, hend, A, Bc);
         load_q_tc<G>(a, w.cu.h, sQ, wg);
         fence_proxy_async_smem();
-        named_sync(kSmBar, 128);
+        named_sync(kSmBar, kTcSoft);
         if (leader) mbar_arrive(smem_u32(q_full));
-        float m = -INFINITY, l = 0.f;
+        float m = -INFINITY, l = 0.f;  // running max (log2 units) and this half's sum, of column col
         int t = 0;
         for (; w.more(); ++t, w.next(a, tab)) {
             const int b = t & 1, s = t % kTcStages;
@@ -402,45 +417,46 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 flags[kFlagOk] = ok;
                 tc_fence_before();
             }
-            named_sync(kSmBar, 128);
+            named_sync(kSmBar, kTcSoft);
             if (!flags[kFlagOk]) break;
             tc_fence_after();
-            float sc[kTcRows];
-            {
-                float v[32];
-                tmem_ld32(tmem + lane_addr + kTcSCol + b * kTcRows, v);
+            float sc[32];
+            tmem_ld32(tmem + lane_addr + kTcSCol + b * kTcRows + 32 * grp, sc);
+            // Raw scores past the segment: -inf (rows 32 grp + i >= cnt).
+            const int valid = cnt - 32 * grp;
+            if (valid < 32) {
 #pragma unroll
-                for (int i = 0; i < 32; ++i) sc[i] = v[i];
-                tmem_ld32(tmem + lane_addr + kTcSCol + b * kTcRows + 32, v);
-#pragma unroll
-                for (int i = 0; i < 32; ++i) sc[32 + i] = v[i];
+                for (int i = 0; i < 32; ++i)
+                    if (i >= valid) sc[i] = -INFINITY;
             }
-            const bool live = L < NC;
-            float mt = -INFINITY;
+            float hm = -INFINITY;
 #pragma unroll
-            for (int r = 0; r < kTcRows; ++r) {
-                sc[r] = (r < cnt) ? sc[r] * cs : -INFINITY;
-                mt = fmaxf(mt, sc[r]);
-            }
-            if (!live) mt = -INFINITY;
+            for (int i = 0; i < 32; ++i) hm = fmaxf(hm, sc[i]);
+            hm = live ? hm * cs : -INFINITY;  // scale > 0: the max of the scaled scores
+            // Exchange the half maxima; a half that tops the running max by kSlack votes
+            // for a rescale (the column needs one exactly when one of its halves does).
+            const bool vote = live && !first && hm > m + kSlack;
+            const unsigned any = __ballot_sync(kFull, vote);
+            if (lane < 16) half_max[grp * kTcMaxCols + col] = hm;
+            if (lane == 0) flags[kFlagVote + sw] = any != 0;
+            named_sync(kSmBar, kTcSoft);
+            const float mt = fmaxf(hm, lane < 16 ? half_max[(grp ^ 1) * kTcMaxCols + col] : -INFINITY);
             if (first) {
                 m = mt;
                 l = 0.f;
             } else {
-                // Lazy rescale: only when a column's tile max tops its running max by kSlack.
-                const bool vote = live && mt > m + kSlack;
-                const unsigned any = __ballot_sync(kFull, vote);
-                if (lane == 0) flags[kFlagVote + (warp & 3)] = any != 0;
-                named_sync(kSmBar, 128);
-                const bool rescale = flags[kFlagVote] | flags[kFlagVote + 1] | flags[kFlagVote + 2] | flags[kFlagVote + 3];
+                bool rescale = false;
+#pragma unroll
+                for (int v = 0; v < 8; ++v) rescale |= flags[kFlagVote + v] != 0;
                 if (rescale) {
+                    const bool mine = live && mt > m + kSlack;
                     float alpha = 1.f;
-                    if (vote) {
+                    if (mine) {
                         alpha = ex2(m - mt);
                         m = mt;
                         l *= alpha;
                     }
-                    if (L < kTcMaxCols) st_a[L] = alpha;
+                    if (grp == 0 && lane < 16) st_alpha[col] = alpha;
                     // O^T of every dimension, column by column, once the product of tile t-1 is done.
                     if (leader) {
                         const bool ok = wait_phase(&o_done[b ^ 1], ((t - 1) >> 1) & 1);
@@ -451,35 +467,38 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         flags[kFlagOk] = ok;
                         tc_fence_before();
                     }
-                    named_sync(kSmBar, 128);
+                    named_sync(kSmBar, kTcSoft);
                     if (!flags[kFlagOk]) break;
                     tc_fence_after();
-                    for (int c0 = 0; c0 < NCpad; c0 += 32) {
+                    if (oc0 < NCpad) {
                         float v[32];
-                        tmem_ld32(tmem + lane_addr + kTcOCol + c0, v);
+                        tmem_ld32(tmem + lane_addr + kTcOCol + oc0, v);
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) v[i] *= (c0 + i < NC) ? st_a[c0 + i] : 1.f;
-                        tmem_st32(tmem + lane_addr + kTcOCol + c0, v);
+                        for (int i = 0; i < 32; ++i) v[i] *= (oc0 + i < NC) ? st_alpha[oc0 + i] : 1.f;
+                        tmem_st32(tmem + lane_addr + kTcOCol + oc0, v);
                     }
                 }
             }
-            // P = 2^(s - m) as bf16 high part and remainder: row L (column L) of the B operand.
-            if (L < NCpad) {
-                const float ref = (m == -INFINITY) ? 0.f : m;
-                unsigned char* ph = sP + b * kTcPBytes + L * 128;
+            // P = 2^(s - m) of this half's 32 rows: a bf16 high part (the top 16 bits)
+            // and the bf16 of the remainder, chunks 4 grp .. 4 grp + 3 of row col
+            // of the B operand (column col's 64 rows, 128 bytes, swizzled).
+            if (lane < 16 && col < NCpad) {
+                const float nm = live ? -m : 0.f;
+                unsigned char* ph = sP + b * kTcPBytes + col * 128;
                 unsigned char* pl = ph + kTcMaxCols * 128;
 #pragma unroll
-                for (int ch = 0; ch < 8; ++ch) {
+                for (int ch = 0; ch < 4; ++ch) {
                     uint32_t hi[4], lo[4];
 #pragma unroll
                     for (int i = 0; i < 4; ++i) {
-                        const float p0 = live ? ex2(sc[8 * ch + 2 * i] - ref) : 0.f;  // 2^-inf = 0 past the segment
-                        const float p1 = live ? ex2(sc[8 * ch + 2 * i + 1] - ref) : 0.f;
+                        const float p0 = live ? ex2(fmaf(sc[8 * ch + 2 * i], cs, nm)) : 0.f;  // 2^-inf = 0
+                        const float p1 = live ? ex2(fmaf(sc[8 * ch + 2 * i + 1], cs, nm)) : 0.f;
                         l += p0 + p1;
-                        hi[i] = pack_bf16(p0, p1);
-                        lo[i] = pack_bf16(p0 - __uint_as_float(hi[i] << 16), p1 - __uint_as_float(hi[i] & 0xffff0000u));
+                        const uint32_t h0 = __float_as_uint(p0) & 0xffff0000u, h1 = __float_as_uint(p1) & 0xffff0000u;
+                        hi[i] = __byte_perm(h0, h1, 0x7632);
+                        lo[i] = pack_bf16(p0 - __uint_as_float(h0), p1 - __uint_as_float(h1));
                     }
-                    const int off = (ch ^ (L & 7)) << 4;
+                    const int off = ((4 * grp + ch) ^ (col & 7)) << 4;
                     *reinterpret_cast<uint4*>(ph + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
                     *reinterpret_cast<uint4*>(pl + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
                 }
@@ -487,7 +506,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             if (cnt < kTcRows) {
                 // V rows past the segment: zeros (their p is 0, but 0 * inf or 0 * nan would not be).
                 unsigned char* v0 = ring + s * kTcStage + 2 * kTcBox;
-                for (int i = wg; i < (kTcRows - cnt) * 16; i += 128) {
+                for (int i = wg; i < (kTcRows - cnt) * 16; i += kTcSoft) {
                     const int r = cnt + (i >> 4), k = i & 15;
                     *reinterpret_cast<uint4*>(v0 + (k >> 3) * kTcBox + r * 128 + ((k & 7) << 4)) =
                         make_uint4(0u, 0u, 0u, 0u);
@@ -495,7 +514,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             }
             fence_proxy_async_smem();
             tc_fence_before();
-            named_sync(kSmBar, 128);
+            named_sync(kSmBar, kTcSoft);
             if (leader) mbar_arrive(smem_u32(&p_full[b]));
             if (!last) continue;
 
@@ -512,11 +531,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     fence_proxy_async_smem();
                 }
             }
-            if (L < NC) {
-                st_m[L] = m;
-                st_l[L] = l;
-            }
-            named_sync(kSmBar, 128);
+            if (lane < 16) half_sum[grp * kTcMaxCols + col] = l;
+            named_sync(kSmBar, kTcSoft);
             // The next segment's Q is in place: its first S product may start. (It must be
             // released before the wait below: the MMA lane issues this tile's O product
             // only after that S product.)
@@ -530,32 +546,33 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 flags[kFlagOk] = ok;
                 tc_fence_before();
             }
-            named_sync(kSmBar, 128);
+            named_sync(kSmBar, kTcSoft);
             if (!flags[kFlagOk]) break;
             tc_fence_after();
             const int bq = h / a.Hkv, g = h - bq * a.Hkv;
             const int64_t slot = (int64_t)c + h;
-            for (int c0 = 0; c0 < NCpad; c0 += 32) {
+            if (oc0 < NCpad) {
                 float v[32];
-                tmem_ld32(tmem + lane_addr + kTcOCol + c0, v);
+                tmem_ld32(tmem + lane_addr + kTcOCol + oc0, v);
 #pragma unroll
                 for (int i = 0; i < 32; ++i) {
-                    const int cc = c0 + i;
+                    const int cc = oc0 + i;
                     if (cc >= NC) break;
                     if (whole) {
-                        const float lc = st_l[cc];
-                        a.out[out_row<G>(a, bq, g, cc) * kHeadDim + L] = lc > 0.f ? v[i] / lc : 0.f;
+                        const float lc = half_sum[cc] + half_sum[kTcMaxCols + cc];
+                        a.out[out_row<G>(a, bq, g, cc) * kHeadDim + dim] = lc > 0.f ? v[i] / lc : 0.f;
                     } else {
-                        a.work_o[(slot * NC + cc) * kHeadDim + L] = v[i];
+                        a.work_o[(slot * NC + cc) * kHeadDim + dim] = v[i];
                     }
                 }
             }
-            if (!whole && L < NC)
-                *reinterpret_cast<float2*>(a.work_ml + (slot * NC + L) * 2) = make_float2(m, l);
+            if (!whole && grp == 0 && live)
+                *reinterpret_cast<float2*>(a.work_ml + (slot * NC + col) * 2) =
+                    make_float2(m, half_sum[col] + half_sum[kTcMaxCols + col]);
             m = -INFINITY;
             l = 0.f;
-            // st_m / st_l are rewritten at the next segment's end, after this one's reads.
-            named_sync(kSmBar, 128);
+            // half_sum is rewritten at the next segment's end, after this one's reads.
+            named_sync(kSmBar, kTcSoft);
         }
     }
 
