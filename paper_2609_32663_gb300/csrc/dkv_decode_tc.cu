@@ -49,25 +49,27 @@ namespace dkv {
 namespace {
 
 constexpr int kTcRows = 64;                    // cache rows per tile
-constexpr int kTcStages = 4;                   // ring stages
+constexpr int kTcStages = 5;                   // ring stages
 constexpr int kTcBox = kTcRows * 128;          // one TMA box: 64 rows x 64 dims of bf16 (8 KB)
 constexpr int kTcStage = 4 * kTcBox;           // K dims 0-63, K dims 64-127, V dims 0-63, V dims 64-127
-constexpr int kTcThreads = 320;                // warps: 0 TMA, 1 MMA, 2-9 softmax and epilogue
+constexpr int kTcThreads = 320;                // warps: 0 TMA, 1 MMA, 2-5 and 6-9 the two softmax groups
 constexpr int kTcSoft = 256;                   // threads of the softmax warps
+constexpr int kTcGroup = 128;                  // threads of one softmax group
 constexpr int kTcQRows = 64;                   // M of the score product: the most columns
 constexpr int kTcQHalf = kTcQRows * 128;       // one 64-dim half of Q (8 KB)
 constexpr int kTcQBytes = 2 * kTcQHalf;        // Q as the A operand: 64 rows x 128 dims
 constexpr int kTcPBytes = 2 * kTcMaxCols * 128;  // one P buffer: high and low parts, 64 columns x 64 rows each
-constexpr int kTcTmemCols = 256;               // S buffers at columns 0 and 64, O at 128
+constexpr int kTcTmemCols = 256;               // S buffers at columns 0 and 64, O of group 0 at 128, of group 1 at 192
 constexpr int kTcSCol = 0, kTcOCol = 128;
-constexpr int kSmBar = 1;                      // named barrier of the softmax warps
+// Named barriers: 1 + g for softmax group g, kBarSoft for both groups, kBarTmem for warps 1-9.
+constexpr int kBarSoft = 3, kBarTmem = 4;
 
 // Shared-memory layout, from a 1024-byte aligned base.
 constexpr int kOffRing = 0;
 constexpr int kOffQ = kOffRing + kTcStages * kTcStage;
 constexpr int kOffP = kOffQ + kTcQBytes;
-constexpr int kOffStats = kOffP + 2 * kTcPBytes;           // half maxima [2][64], half sums [2][64], alpha[64] (floats)
-constexpr int kOffFlags = kOffStats + 5 * kTcMaxCols * 4;  // int[16]
+constexpr int kOffStats = kOffP + 2 * kTcPBytes;           // per group: max [2][64], sum [2][64], alpha [2][64] (floats)
+constexpr int kOffFlags = kOffStats + 6 * kTcMaxCols * 4;  // int[16]
 constexpr int kOffBars = kOffFlags + 16 * 4;               // uint64 barriers
 // full[S], empty[S], s_full[2], p_full[2], o_done[2], q_full, fin
 constexpr int kNumBars = 2 * kTcStages + 8;
@@ -78,12 +80,13 @@ __host__ __device__ constexpr int tc_smem_bytes(int B) { return kTcAlign + kOffT
 static_assert(tc_smem_bytes(kMaxB) <= 227 * 1024, "fits the opt-in shared memory of one CTA");
 
 // Flag slots.
-constexpr int kFlagVote = 0;      // [8] per-warp rescale votes of the softmax warps
+constexpr int kFlagVote = 0;      // [2][4] per-warp rescale votes of each softmax group
 constexpr int kFlagAbort = 8;     // a bounded wait ran out
-constexpr int kFlagOk = 9;        // result of the leader's wait, for the softmax warps
-constexpr int kFlagIssued = 10;   // tiles the TMA lane issued
-constexpr int kFlagConsumed = 11;  // tiles whose copies the MMA lane saw land
-constexpr int kFlagMmaLast = 12;  // the MMA lane issued products (fin must be awaited before freeing TMEM)
+constexpr int kFlagOk = 9;        // [2] result of a group leader's wait, for its group (10: group 1)
+constexpr int kFlagSegOk = 11;    // no wait ran out before a segment's end (for both groups)
+constexpr int kFlagIssued = 12;   // tiles the TMA lane issued
+constexpr int kFlagConsumed = 13;  // tiles whose copies the MMA lane saw land
+constexpr int kFlagMmaLast = 14;  // the MMA lane issued products (fin must be awaited before freeing TMEM)
 
 // ------------------------------------------------------------ tcgen05 wrappers
 // Shared-memory matrix descriptor: start address, leading and stride byte
@@ -229,16 +232,18 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     unsigned char* ring = sm + kOffRing;
     unsigned char* sQ = sm + kOffQ;
     unsigned char* sP = sm + kOffP;
-    float* st_m = reinterpret_cast<float*>(sm + kOffStats);
+    float* g_max = reinterpret_cast<float*>(sm + kOffStats);  // [2][64] running max of each group, at a segment's end
+    float* g_sum = g_max + 2 * kTcMaxCols;                     // [2][64] its sum
+    float* g_alpha = g_sum + 2 * kTcMaxCols;                   // [2][64] rescale factors of a tile
     volatile int* flags = reinterpret_cast<volatile int*>(sm + kOffFlags);
     uint64_t* bars = reinterpret_cast<uint64_t*>(sm + kOffBars);
-    uint64_t* full = bars;
-    uint64_t* empty = bars + kTcStages;
-    uint64_t* s_full = bars + 2 * kTcStages;
-    uint64_t* p_full = s_full + 2;
-    uint64_t* o_done = p_full + 2;
-    uint64_t* q_full = o_done + 2;
-    uint64_t* fin = q_full + 1;
+    uint64_t* full = bars;                    // [S] the stage's copies landed
+    uint64_t* empty = bars + kTcStages;       // [S] the stage's products are done
+    uint64_t* s_full = bars + 2 * kTcStages;  // [2] S of tile t (buffer t & 1) is done
+    uint64_t* p_full = s_full + 2;            // [2] P of tile t is written
+    uint64_t* o_done = p_full + 2;            // [2] the O product of tile t is done
+    uint64_t* q_full = o_done + 2;            // the segment's Q is in place
+    uint64_t* fin = q_full + 1;               // drain after a timeout
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + kOffTmem);
     const SeqTable tab = seq_table_at(sm + kOffTable, a);
 
@@ -271,22 +276,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (A >= Bc) return;  // uniform: this CTA has no rows (no TMEM taken yet)
     const int hfirst = slab_containing(a, tab, NHl, A);
     const int hend = slab_containing(a, tab, NHl, Bc - 1) + 1;
-
-    if (warp == 1) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
-                     "r"(kTcTmemCols));
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
-    }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t tmem = *tmem_slot;
     const int NC = a.NC;
     const int NCpad = (NC + 15) & ~15;
     const float cs = a.qscale;
+    uint32_t tmem = 0;
 
     if (warp == 0) {
         // ---------------------------------------------------------------- TMA
+        // Starts at once: the copies need no TMEM.
         if (lane == 0) {
             const uint64_t pol = evict_first_policy();
             TileWalk w;
@@ -312,27 +309,42 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             }
             flags[kFlagIssued] = t;
         }
-    } else if (warp == 1) {
+    } else {
+        if (warp == 1) {
+            asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                         "r"(kTcTmemCols));
+            asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+        }
+        tc_fence_before();
+        named_sync(kBarTmem, kTcThreads - 32);
+        tc_fence_after();
+        tmem = *tmem_slot;
+    }
+
+    if (warp == 1) {
         // ---------------------------------------------------------------- MMA
         if (lane == 0) {
             const uint32_t id1 = idesc(kTcQRows, kTcRows, 0, 0);
             const uint32_t id2 = idesc(128, NCpad, 1, 0);
             TileWalk w;
             w.begin(a, tab, hfirst, hend, A, Bc);
-            int t = 0, seg = 0;
-            bool prev_first = false, issued = false, ok = true;
-            // O^T += V^T P for tile u (its stage's V, its P buffer), then release the stage.
-            auto mma2 = [&](int u, bool first_of_seg) -> bool {
+            int t = 0, seg = 0, seg_start = 0, prev_seg_start = 0;
+            bool issued = false, ok = true;
+            // O^T += V^T P for tile u into its group's accumulator (u & 1), then
+            // release the stage. A group's first tile of a segment starts it afresh.
+            auto mma2 = [&](int u, int u_seg_start) -> bool {
                 const int b = u & 1, s = u % kTcStages;
                 if (!wait_phase(&p_full[b], (u >> 1) & 1)) return false;
                 tc_fence_after();
                 const uint32_t v0 = smem_u32(ring + s * kTcStage + 2 * kTcBox);
                 const uint32_t p0 = smem_u32(sP + b * kTcPBytes);
+                const uint32_t o = tmem + kTcOCol + b * kTcMaxCols;
+                const uint32_t fresh = (u - u_seg_start) < 2;
 #pragma unroll
                 for (int k = 0; k < kTcRows / 16; ++k) {
                     const uint64_t av = sdesc(v0 + k * 2048, kTcBox, 1024);
-                    umma(tmem + kTcOCol, av, sdesc(p0 + k * 32, 16, 1024), id2, (first_of_seg && k == 0) ? 0u : 1u);
-                    umma(tmem + kTcOCol, av, sdesc(p0 + kTcMaxCols * 128 + k * 32, 16, 1024), id2, 1u);
+                    umma(o, av, sdesc(p0 + k * 32, 16, 1024), id2, (fresh && k == 0) ? 0u : 1u);
+                    umma(o, av, sdesc(p0 + kTcMaxCols * 128 + k * 32, 16, 1024), id2, 1u);
                 }
                 umma_commit(smem_u32(&o_done[b]));
                 umma_commit(smem_u32(&empty[s]));
@@ -350,9 +362,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     break;
                 }
                 flags[kFlagConsumed] = t + 1;
-                if (first && !wait_phase(q_full, seg++ & 1)) {
-                    ok = false;
-                    break;
+                if (first) {
+                    if (!wait_phase(q_full, seg++ & 1)) {
+                        ok = false;
+                        break;
+                    }
+                    prev_seg_start = seg_start;
+                    seg_start = t;
                 }
                 tc_fence_after();
                 // S^T[64 x 64] = Q[64 x 128] K^T: k-steps of 16 dims (+32 B inside a 64-dim half).
@@ -363,162 +379,168 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                          sdesc(k0 + (k >> 2) * kTcBox + (k & 3) * 32, 16, 1024), id1, k > 0 ? 1u : 0u);
                 umma_commit(smem_u32(&s_full[b]));
                 issued = true;
-                if (t > 0 && !mma2(t - 1, prev_first)) {
+                if (t > 0 && !mma2(t - 1, first ? prev_seg_start : seg_start)) {
                     ok = false;
                     break;
                 }
-                prev_first = first;
             }
-            if (ok && t > 0 && !mma2(t - 1, prev_first)) ok = false;
+            if (ok && t > 0 && !mma2(t - 1, seg_start)) ok = false;
             if (!ok) {
                 atomicOr(a.status, 0x2 /* DKV_DEV_TMA_TIMEOUT */);
                 flags[kFlagAbort] = 1;
             }
             flags[kFlagMmaLast] = issued ? 1 : 0;
         }
-    } else {
-        // ---------------------------------------------------------------- softmax and epilogue
-        const int sw = warp - 2;                    // 0..7
-        const int grp = sw >> 2;                    // row half of the tile (scores), column chunk (O)
-        const int quarter = warp & 3;               // TMEM lane quarter this warp may access
-        const int wg = tid - 64;                    // 0..255 within the softmax warps
-        const bool leader = wg == 0;
+    } else if (warp >= 2) {
+        // ---------------------------------------------------------------- softmax groups and epilogue
+        // Group gi takes the tiles t with t % 2 == gi, with its own running max and
+        // sum of each column and its own O accumulator; the two are merged at the
+        // end of a segment. Thread (quarter, lane < 16) owns column 16 quarter + lane
+        // (TMEM lane 32 quarter + lane of S^T, all 64 rows of a tile); for O, thread
+        // (quarter, lane) owns dimension 32 quarter + lane.
+        const int gi = (warp - 2) >> 2;
+        const int quarter = warp & 3;
+        const int gt = tid - 64 - kTcGroup * gi;   // 0..127 within the group
+        const int st = tid - 64;                    // 0..255 within both groups
+        const bool gleader = gt == 0, leader = st == 0;
+        const int gbar = 1 + gi;
         const uint32_t lane_addr = (uint32_t)(32 * quarter) << 16;
-        // Scores: column c = 16 quarter + lane (lanes 0-15), rows 32 grp .. 32 grp + 31.
         const int col = 16 * quarter + lane;
         const bool live = lane < 16 && col < NC;
-        float* half_max = st_m;                     // [2][64]
-        float* half_sum = st_m + 2 * kTcMaxCols;    // [2][64]
-        float* st_alpha = st_m + 4 * kTcMaxCols;    // [64]
-        // O: dimension d = 32 quarter + lane, columns 32 grp .. 32 grp + 31.
         const int dim = 32 * quarter + lane;
-        const int oc0 = 32 * grp;
+        const uint32_t my_o = tmem + lane_addr + kTcOCol + gi * kTcMaxCols;
         pdl_wait();  // q and the outputs belong to the previous kernel's epoch
         TileWalk w;
         w.begin(a, tab, hfirst, hend, A, Bc);
-        load_q_tc<G>(a, w.cu.h, sQ, wg);
+        load_q_tc<G>(a, w.cu.h, sQ, st);
         fence_proxy_async_smem();
-        named_sync(kSmBar, kTcSoft);
+        named_sync(kBarSoft, kTcSoft);
         if (leader) mbar_arrive(smem_u32(q_full));
-        float m = -INFINITY, l = 0.f;  // running max (log2 units) and this half's sum, of column col
-        int t = 0;
-        for (; w.more(); ++t, w.next(a, tab)) {
-            const int b = t & 1, s = t % kTcStages;
-            const int cnt = w.cnt();
-            const bool first = w.first(), last = w.last();
-            // The tile's scores, and the end of the product that last read P buffer b.
-            if (leader) {
-                bool ok = !flags[kFlagAbort] && wait_phase(&s_full[b], (t >> 1) & 1);
-                if (ok && t >= 2) ok = wait_phase(&o_done[b], ((t - 2) >> 1) & 1);
-                if (!ok) {
-                    atomicOr(a.status, 0x2 /* DKV_DEV_TMA_TIMEOUT */);
-                    flags[kFlagAbort] = 1;
-                }
-                flags[kFlagOk] = ok;
-                tc_fence_before();
-            }
-            named_sync(kSmBar, kTcSoft);
-            if (!flags[kFlagOk]) break;
-            tc_fence_after();
-            float sc[32];
-            tmem_ld32(tmem + lane_addr + kTcSCol + b * kTcRows + 32 * grp, sc);
-            // Raw scores past the segment: -inf (rows 32 grp + i >= cnt).
-            const int valid = cnt - 32 * grp;
-            if (valid < 32) {
-#pragma unroll
-                for (int i = 0; i < 32; ++i)
-                    if (i >= valid) sc[i] = -INFINITY;
-            }
-            float hm = -INFINITY;
-#pragma unroll
-            for (int i = 0; i < 32; ++i) hm = fmaxf(hm, sc[i]);
-            hm = live ? hm * cs : -INFINITY;  // scale > 0: the max of the scaled scores
-            // Exchange the half maxima; a half that tops the running max by kSlack votes
-            // for a rescale (the column needs one exactly when one of its halves does).
-            const bool vote = live && !first && hm > m + kSlack;
-            const unsigned any = __ballot_sync(kFull, vote);
-            if (lane < 16) half_max[grp * kTcMaxCols + col] = hm;
-            if (lane == 0) flags[kFlagVote + sw] = any != 0;
-            named_sync(kSmBar, kTcSoft);
-            const float mt = fmaxf(hm, lane < 16 ? half_max[(grp ^ 1) * kTcMaxCols + col] : -INFINITY);
-            if (first) {
-                m = mt;
+        float m = -INFINITY, l = 0.f;  // this group's running max (log2 units) and sum of column col
+        int t = 0, seg_start = 0;
+        int last_mine = -1;            // this group's last tile of the current segment
+        bool stop = false;             // set at a segment's end, the same in both groups
+        // After a wait runs out a group keeps walking the tiles (without work) so that
+        // both groups meet at every segment's end: a named barrier has no bound.
+        for (; w.more() && !stop; ++t, w.next(a, tab)) {
+            if (w.first()) {
+                seg_start = t;
+                last_mine = -1;
+                m = -INFINITY;
                 l = 0.f;
-            } else {
-                bool rescale = false;
-#pragma unroll
-                for (int v = 0; v < 8; ++v) rescale |= flags[kFlagVote + v] != 0;
-                if (rescale) {
-                    const bool mine = live && mt > m + kSlack;
-                    float alpha = 1.f;
-                    if (mine) {
-                        alpha = ex2(m - mt);
-                        m = mt;
-                        l *= alpha;
+            }
+            const bool last = w.last();
+            if ((t & 1) == gi) {
+                const int b = gi, s = t % kTcStages;
+                const int cnt = w.cnt();
+                const bool gfirst = t - seg_start < 2;  // the group's first tile of the segment
+                last_mine = t;
+                // The tile's scores, and the end of the group's previous O product
+                // (it read P buffer b, and rescaling O needs it done).
+                if (gleader) {
+                    bool ok = !flags[kFlagAbort] && wait_phase(&s_full[b], (t >> 1) & 1);
+                    if (ok && t >= 2) ok = wait_phase(&o_done[b], ((t - 2) >> 1) & 1);
+                    if (!ok) {
+                        atomicOr(a.status, 0x2 /* DKV_DEV_TMA_TIMEOUT */);
+                        flags[kFlagAbort] = 1;
                     }
-                    if (grp == 0 && lane < 16) st_alpha[col] = alpha;
-                    // O^T of every dimension, column by column, once the product of tile t-1 is done.
-                    if (leader) {
-                        const bool ok = wait_phase(&o_done[b ^ 1], ((t - 1) >> 1) & 1);
-                        if (!ok) {
-                            atomicOr(a.status, 0x2 /* DKV_DEV_TMA_TIMEOUT */);
-                            flags[kFlagAbort] = 1;
-                        }
-                        flags[kFlagOk] = ok;
-                        tc_fence_before();
-                    }
-                    named_sync(kSmBar, kTcSoft);
-                    if (!flags[kFlagOk]) break;
+                    flags[kFlagOk + gi] = ok;
+                    tc_fence_before();
+                }
+                named_sync(gbar, kTcGroup);
+                if (!flags[kFlagOk + gi]) {
+                    named_sync(gbar, kTcGroup);  // the flag is rewritten at the group's next tile
+                } else {
                     tc_fence_after();
-                    if (oc0 < NCpad) {
-                        float v[32];
-                        tmem_ld32(tmem + lane_addr + kTcOCol + oc0, v);
+                    float sc[kTcRows];
+                    tmem_ld32(tmem + lane_addr + kTcSCol + b * kTcRows, *reinterpret_cast<float(*)[32]>(sc));
+                    tmem_ld32(tmem + lane_addr + kTcSCol + b * kTcRows + 32, *reinterpret_cast<float(*)[32]>(sc + 32));
+                    if (cnt < kTcRows) {
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) v[i] *= (oc0 + i < NC) ? st_alpha[oc0 + i] : 1.f;
-                        tmem_st32(tmem + lane_addr + kTcOCol + oc0, v);
+                        for (int i = 0; i < kTcRows; ++i)
+                            if (i >= cnt) sc[i] = -INFINITY;  // rows past the segment
                     }
-                }
-            }
-            // P = 2^(s - m) of this half's 32 rows: a bf16 high part (the top 16 bits)
-            // and the bf16 of the remainder, chunks 4 grp .. 4 grp + 3 of row col
-            // of the B operand (column col's 64 rows, 128 bytes, swizzled).
-            if (lane < 16 && col < NCpad) {
-                const float nm = live ? -m : 0.f;
-                unsigned char* ph = sP + b * kTcPBytes + col * 128;
-                unsigned char* pl = ph + kTcMaxCols * 128;
+                    float mt = -INFINITY;
 #pragma unroll
-                for (int ch = 0; ch < 4; ++ch) {
-                    uint32_t hi[4], lo[4];
+                    for (int i = 0; i < kTcRows; ++i) mt = fmaxf(mt, sc[i]);
+                    mt = live ? mt * cs : -INFINITY;  // scale > 0: the max of the scaled scores
+                    if (gfirst) {
+                        m = mt;
+                        l = 0.f;
+                    } else {
+                        // Lazy rescale: only when a column's tile max tops its running max by kSlack.
+                        const bool vote = live && mt > m + kSlack;
+                        const unsigned any = __ballot_sync(kFull, vote);
+                        if (lane == 0) flags[kFlagVote + 4 * gi + quarter] = any != 0;
+                        named_sync(gbar, kTcGroup);
+                        const bool rescale = flags[kFlagVote + 4 * gi] | flags[kFlagVote + 4 * gi + 1] |
+                                             flags[kFlagVote + 4 * gi + 2] | flags[kFlagVote + 4 * gi + 3];
+                        if (rescale) {
+                            float alpha = 1.f;
+                            if (vote) {
+                                alpha = ex2(m - mt);
+                                m = mt;
+                                l *= alpha;
+                            }
+                            if (lane < 16) g_alpha[gi * kTcMaxCols + col] = alpha;
+                            named_sync(gbar, kTcGroup);
+                            // The group's O (its previous product is done: waited above).
+                            for (int c0 = 0; c0 < NCpad; c0 += 32) {
+                                float v[32];
+                                tmem_ld32(my_o + c0, v);
 #pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        const float p0 = live ? ex2(fmaf(sc[8 * ch + 2 * i], cs, nm)) : 0.f;  // 2^-inf = 0
-                        const float p1 = live ? ex2(fmaf(sc[8 * ch + 2 * i + 1], cs, nm)) : 0.f;
-                        l += p0 + p1;
-                        const uint32_t h0 = __float_as_uint(p0) & 0xffff0000u, h1 = __float_as_uint(p1) & 0xffff0000u;
-                        hi[i] = __byte_perm(h0, h1, 0x7632);
-                        lo[i] = pack_bf16(p0 - __uint_as_float(h0), p1 - __uint_as_float(h1));
+                                for (int i = 0; i < 32; ++i)
+                                    v[i] *= (c0 + i < NC) ? g_alpha[gi * kTcMaxCols + c0 + i] : 1.f;
+                                tmem_st32(my_o + c0, v);
+                            }
+                        }
                     }
-                    const int off = ((4 * grp + ch) ^ (col & 7)) << 4;
-                    *reinterpret_cast<uint4*>(ph + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-                    *reinterpret_cast<uint4*>(pl + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+                    // P = 2^(s - m): a bf16 high part (the top 16 bits) and the bf16 of
+                    // the remainder, row col of the B operand (64 rows, 128 bytes, swizzled).
+                    if (lane < 16 && col < NCpad) {
+                        const float nm = live ? -m : 0.f;
+                        unsigned char* ph = sP + b * kTcPBytes + col * 128;
+                        unsigned char* pl = ph + kTcMaxCols * 128;
+#pragma unroll
+                        for (int ch = 0; ch < 8; ++ch) {
+                            uint32_t hi[4], lo[4];
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) {
+                                const float p0 = live ? ex2(fmaf(sc[8 * ch + 2 * i], cs, nm)) : 0.f;  // 2^-inf = 0
+                                const float p1 = live ? ex2(fmaf(sc[8 * ch + 2 * i + 1], cs, nm)) : 0.f;
+                                l += p0 + p1;
+                                const uint32_t h0 = __float_as_uint(p0) & 0xffff0000u;
+                                const uint32_t h1 = __float_as_uint(p1) & 0xffff0000u;
+                                hi[i] = __byte_perm(h0, h1, 0x7632);
+                                lo[i] = pack_bf16(p0 - __uint_as_float(h0), p1 - __uint_as_float(h1));
+                            }
+                            const int off = (ch ^ (col & 7)) << 4;
+                            *reinterpret_cast<uint4*>(ph + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+                            *reinterpret_cast<uint4*>(pl + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+                        }
+                    }
+                    if (cnt < kTcRows) {
+                        // V rows past the segment: zeros (their p is 0, but 0 * inf or 0 * nan would not be).
+                        unsigned char* v0 = ring + s * kTcStage + 2 * kTcBox;
+                        for (int i = gt; i < (kTcRows - cnt) * 16; i += kTcGroup) {
+                            const int r = cnt + (i >> 4), k = i & 15;
+                            *reinterpret_cast<uint4*>(v0 + (k >> 3) * kTcBox + r * 128 + ((k & 7) << 4)) =
+                                make_uint4(0u, 0u, 0u, 0u);
+                        }
+                    }
+                    fence_proxy_async_smem();
+                    tc_fence_before();
+                    named_sync(gbar, kTcGroup);
+                    if (gleader) mbar_arrive(smem_u32(&p_full[b]));
                 }
             }
-            if (cnt < kTcRows) {
-                // V rows past the segment: zeros (their p is 0, but 0 * inf or 0 * nan would not be).
-                unsigned char* v0 = ring + s * kTcStage + 2 * kTcBox;
-                for (int i = wg; i < (kTcRows - cnt) * 16; i += kTcSoft) {
-                    const int r = cnt + (i >> 4), k = i & 15;
-                    *reinterpret_cast<uint4*>(v0 + (k >> 3) * kTcBox + r * 128 + ((k & 7) << 4)) =
-                        make_uint4(0u, 0u, 0u, 0u);
-                }
-            }
-            fence_proxy_async_smem();
-            tc_fence_before();
-            named_sync(kSmBar, kTcSoft);
-            if (leader) mbar_arrive(smem_u32(&p_full[b]));
             if (!last) continue;
 
-            // ---- end of a segment: the next segment's Q, then this one's output or partial.
+            // ---- end of a segment, both groups: the next segment's Q, then the merge of
+            // the two groups' states and this segment's output or partial.
+            if (leader) flags[kFlagSegOk] = !flags[kFlagAbort];
+            named_sync(kBarSoft, kTcSoft);  // every S product of the segment was seen done by its group
+            const bool seg_ok = flags[kFlagSegOk];
             const int h = w.cu.h, p0h = w.cu.p0, p1h = w.cu.p0 + w.cu.n_h;
             const bool whole = w.cu.s0 == p0h && w.cu.s1 == p1h;
             bool has_next = false;
@@ -527,52 +549,62 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 nx.next(a, tab);
                 has_next = nx.more();
                 if (has_next) {
-                    load_q_tc<G>(a, nx.cu.h, sQ, wg);
+                    load_q_tc<G>(a, nx.cu.h, sQ, st);
                     fence_proxy_async_smem();
                 }
             }
-            if (lane < 16) half_sum[grp * kTcMaxCols + col] = l;
-            named_sync(kSmBar, kTcSoft);
+            const bool has0 = (t - seg_start >= 1) || ((seg_start & 1) == 0);  // group 0 had a tile here
+            const bool has1 = (t - seg_start >= 1) || ((seg_start & 1) == 1);
+            if (lane < 16) {
+                g_max[gi * kTcMaxCols + col] = m;
+                g_sum[gi * kTcMaxCols + col] = l;
+            }
+            named_sync(kBarSoft, kTcSoft);
             // The next segment's Q is in place: its first S product may start. (It must be
-            // released before the wait below: the MMA lane issues this tile's O product
-            // only after that S product.)
+            // released before the waits below: the MMA lane issues this segment's last O
+            // product only after that S product.)
             if (leader && has_next) mbar_arrive(smem_u32(q_full));
-            if (leader) {
-                const bool ok = wait_phase(&o_done[b], (t >> 1) & 1);
-                if (!ok) {
+            if (gleader) {
+                bool ok = seg_ok;
+                if (ok && last_mine >= 0) ok = wait_phase(&o_done[gi], (last_mine >> 1) & 1);
+                if (seg_ok && !ok) {
                     atomicOr(a.status, 0x2 /* DKV_DEV_TMA_TIMEOUT */);
                     flags[kFlagAbort] = 1;
                 }
-                flags[kFlagOk] = ok;
+                flags[kFlagOk + gi] = ok;
                 tc_fence_before();
             }
-            named_sync(kSmBar, kTcSoft);
-            if (!flags[kFlagOk]) break;
+            named_sync(kBarSoft, kTcSoft);
+            const bool merge_ok = flags[kFlagOk] && flags[kFlagOk + 1];
+            stop = !merge_ok;
             tc_fence_after();
+            // Merge: group gi writes the columns 32 gi .. 32 gi + 31 of every dimension.
+            const int oc0 = 32 * gi;
             const int bq = h / a.Hkv, g = h - bq * a.Hkv;
             const int64_t slot = (int64_t)c + h;
-            if (oc0 < NCpad) {
-                float v[32];
-                tmem_ld32(tmem + lane_addr + kTcOCol + oc0, v);
+            if (merge_ok && oc0 < NCpad) {
+                float v0[32], v1[32];
+                tmem_ld32(tmem + lane_addr + kTcOCol + oc0, v0);
+                tmem_ld32(tmem + lane_addr + kTcOCol + kTcMaxCols + oc0, v1);
 #pragma unroll
                 for (int i = 0; i < 32; ++i) {
                     const int cc = oc0 + i;
                     if (cc >= NC) break;
+                    const float m0 = has0 ? g_max[cc] : -INFINITY, m1 = has1 ? g_max[kTcMaxCols + cc] : -INFINITY;
+                    const float M = fmaxf(m0, m1);
+                    const float f0 = has0 ? ex2(m0 - M) : 0.f, f1 = has1 ? ex2(m1 - M) : 0.f;
+                    const float o = (has0 ? f0 * v0[i] : 0.f) + (has1 ? f1 * v1[i] : 0.f);
+                    const float L = (has0 ? f0 * g_sum[cc] : 0.f) + (has1 ? f1 * g_sum[kTcMaxCols + cc] : 0.f);
                     if (whole) {
-                        const float lc = half_sum[cc] + half_sum[kTcMaxCols + cc];
-                        a.out[out_row<G>(a, bq, g, cc) * kHeadDim + dim] = lc > 0.f ? v[i] / lc : 0.f;
+                        a.out[out_row<G>(a, bq, g, cc) * kHeadDim + dim] = L > 0.f ? o / L : 0.f;
                     } else {
-                        a.work_o[(slot * NC + cc) * kHeadDim + dim] = v[i];
+                        a.work_o[(slot * NC + cc) * kHeadDim + dim] = o;
+                        if (dim == 0) *reinterpret_cast<float2*>(a.work_ml + (slot * NC + cc) * 2) = make_float2(M, L);
                     }
                 }
             }
-            if (!whole && grp == 0 && live)
-                *reinterpret_cast<float2*>(a.work_ml + (slot * NC + col) * 2) =
-                    make_float2(m, half_sum[col] + half_sum[kTcMaxCols + col]);
-            m = -INFINITY;
-            l = 0.f;
-            // half_sum is rewritten at the next segment's end, after this one's reads.
-            named_sync(kSmBar, kTcSoft);
+            // g_max / g_sum are rewritten at the next segment's end, after these reads.
+            named_sync(kBarSoft, kTcSoft);
         }
     }
 
