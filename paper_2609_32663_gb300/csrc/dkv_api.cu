@@ -180,7 +180,7 @@ dkv_status plan_configs(dkv_plan* p)
     }
     p->cols_cap = dkv::kMaxCols;
     const int64_t NHl = (int64_t)p->B * p->s.H_kv;
-    p->work = dkv::workspace_layout(ctas + NHl, dkv::kTcMaxCols, warp_records, dkv::kMaxCols, NHl);
+    p->work = dkv::workspace_layout(ctas + NHl, dkv::kTcMaxCols, warp_records, dkv::kMaxCols);
     return DKV_OK;
 }
 
@@ -606,7 +606,6 @@ dkv_status decode_args(const dkv_plan* p, int32_t layer, const void* q, const vo
     a->work_ml = p->d_work + p->work.work_ml;
     a->warp_o = p->d_work + p->work.warp_o;
     a->warp_ml = p->d_work + p->work.warp_ml;
-    a->tc_bounds = reinterpret_cast<int32_t*>(p->d_work + p->work.bounds);
     if (!aligned16(a->work_o) || !aligned16(a->work_ml) || !aligned16(a->warp_o) || !aligned16(a->warp_ml))
         return fail(DKV_ERR_INVALID_ARG, "split-K workspace regions are not 16-byte aligned");
     a->out = out;
@@ -673,7 +672,7 @@ dkv_status dkv_decode_multi(const dkv_plan* p, int32_t layer, const void* q, int
     a.NC = num_queries * p->G;
     if (a.NC > dkv::kMaxCols) {
         // More columns than the mma.sync kernels' accumulator registers hold: the
-        // tcgen05 kernel (accumulators in TMEM) and its combine launch.
+        // tcgen05 kernel (accumulators in TMEM).
         a.nctas = p->cfg_tc.nctas;
         dkv::CacheMaps maps;
         const cudaError_t e = dkv::make_cache_maps(a.Kc, a.Vc, p->total_rows, &maps, fault("copy"), 64);

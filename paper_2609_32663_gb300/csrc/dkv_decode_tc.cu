@@ -4,41 +4,49 @@
 // (queries x heads of a KV head's group) per slab.
 //
 // Work split: the layer's rows (every slab end to end, plus the rows appended in
-// earlier steps) are cut into equal contiguous CTA ranges (one CTA per SM), as in
-// the other decode kernels; a CTA walks its range in tiles of 64 rows, slab
-// segment by slab segment. Per tile, one pipeline per CTA:
+// earlier steps) are cut into equal contiguous CTA ranges (one CTA per SM, a
+// cooperative launch, so every CTA is resident at once), as in the other decode
+// kernels; a CTA walks its range in tiles of 64 rows, slab segment by slab
+// segment (a segment: the part of one slab inside the CTA's range).
 //
-//   warp 0 (one lane)   TMA: the tile's K and V rows as four 2-D boxes
-//                       (64 rows x 64 dims, 128-byte swizzle) into a 4-stage ring.
+//   warp 0 (one lane)   TMA: a tile's K rows and V rows, each as two 2-D boxes
+//                       (64 rows x 64 dims, 128-byte swizzle), into separate
+//                       rings (4 K stages, 6 V stages): a K stage is released as
+//                       soon as its score product is done, a V stage only after
+//                       its output product, so V is the deeper ring.
 //   warp 1 (one lane)   MMA: S^T = Q K^T  (M = 64 query-column rows of Q, zero
 //                       past the last column, N = 64 cache rows, K = 128 dims;
-//                       8 MMAs) into one of two TMEM score buffers, then, one tile
-//                       behind, O^T += V^T P  (M = 128 dims, N = the columns
-//                       rounded up to 16, K = 64 rows; V^T read MN-major from the
-//                       same stage; P as a bf16 high part and remainder, two MMAs
-//                       per k-step) into the TMEM output accumulator.
-//   warps 2-9           softmax: with M = 64, row c of S^T (column c) sits in
-//                       TMEM lane 32 (c / 16) + c % 16. Warps 2-5 take rows 0-31
-//                       of the tile and warps 6-9 rows 32-63, one column a thread
-//                       (lanes 0-15 of each warp): half-tile max, exchanged once
-//                       per tile, lazily rescaled running max (a column's max
+//                       8 MMAs) into one of four TMEM score buffers, running up
+//                       to four tiles ahead of O^T += V^T P  (M = 128 dims, N =
+//                       the columns rounded up to 16, K = 64 rows; V^T read
+//                       MN-major from its stage; P as a bf16 high part and
+//                       remainder, two MMAs per k-step) into the TMEM output
+//                       accumulator of the tile's softmax group.
+//   warps 2-5, 6-9      two softmax groups; group g takes the tiles t with
+//                       t % 2 == g, with its own running max and sum of every
+//                       column and its own O accumulator (merged at a segment's
+//                       end). With M = 64, row c of S^T (column c) sits in TMEM
+//                       lane 32 (c / 16) + c % 16: thread (quarter, lane < 16)
+//                       owns column 16 quarter + lane, all 64 rows of a tile:
+//                       tile max, lazily rescaled running max (a column's max
 //                       moves only when a score tops it by kSlack; O is then
 //                       rescaled in TMEM), P = 2^(s - m) written to shared memory
-//                       as the B operand of the next product, V rows past a
-//                       segment zeroed. At a segment's end the same warps read
-//                       O^T (thread d of a warp quarter owns dimension d, TMEM lane
-//                       d; the two halves take 32 columns each) and write the
-//                       slab's output, or the CTA's partial (m, l, o) of each
-//                       column when the slab continues in another CTA.
+//                       as the B operand of the output product, V rows past a
+//                       segment zeroed. For O, thread (quarter, lane) owns
+//                       dimension 32 quarter + lane (TMEM lane).
 //
-// Slabs that span several CTAs are merged by decode_tc_combine_kernel, a separate
-// launch with one CTA per (slab, column): with up to 64 columns a slab's partials
-// are up to 64 x 19 records at the 128K context, too many for the last CTA of
-// the slab to merge alone in time.
+// A slab wholly inside one CTA is written out at its segment's end. Otherwise
+// each CTA of the slab writes its partial (m, l, o of every column) and counts
+// itself in; once the CTA's range is done it waits (bounded) until all the
+// slab's CTAs have counted in, then merges its share of the slab's columns
+// (CTA k of the slab's nct CTAs takes columns k NC / nct .. (k+1) NC / nct):
+// the merge is spread over the slab's CTAs instead of falling on the last one.
 //
-// Every wait is bounded (polls and 2 s); a wait that runs out sets
-// DKV_DEV_TMA_TIMEOUT, the roles stop, the copies and products in flight are
-// drained with the same bound, and TMEM is freed before the CTA exits.
+// Every wait is bounded (polls and 2 s). A wait that runs out sets a
+// DKV_DEV_* bit, the roles stop (the softmax groups keep walking the tiles,
+// without work, so that they still meet at every named barrier), the copies and
+// products in flight are drained with the same bound, and TMEM is freed before
+// the CTA exits.
 #include "dkv_decode_common.cuh"
 
 #include <cuda.h>
@@ -49,9 +57,10 @@ namespace dkv {
 namespace {
 
 constexpr int kTcRows = 64;                    // cache rows per tile
-constexpr int kTcStages = 5;                   // ring stages
+constexpr int kKStages = 4;                    // K ring stages
+constexpr int kVStages = 6;                    // V ring stages
 constexpr int kTcBox = kTcRows * 128;          // one TMA box: 64 rows x 64 dims of bf16 (8 KB)
-constexpr int kTcStage = 4 * kTcBox;           // K dims 0-63, K dims 64-127, V dims 0-63, V dims 64-127
+constexpr int kTcHalfTile = 2 * kTcBox;        // K (or V) rows of one tile: dims 0-63, then 64-127
 constexpr int kTcThreads = 320;                // warps: 0 TMA, 1 MMA, 2-5 and 6-9 the two softmax groups
 constexpr int kTcSoft = 256;                   // threads of the softmax warps
 constexpr int kTcGroup = 128;                  // threads of one softmax group
@@ -59,20 +68,22 @@ constexpr int kTcQRows = 64;                   // M of the score product: the mo
 constexpr int kTcQHalf = kTcQRows * 128;       // one 64-dim half of Q (8 KB)
 constexpr int kTcQBytes = 2 * kTcQHalf;        // Q as the A operand: 64 rows x 128 dims
 constexpr int kTcPBytes = 2 * kTcMaxCols * 128;  // one P buffer: high and low parts, 64 columns x 64 rows each
-constexpr int kTcTmemCols = 256;               // S buffers at columns 0 and 64, O of group 0 at 128, of group 1 at 192
-constexpr int kTcSCol = 0, kTcOCol = 128;
+constexpr int kSBufs = 4;                      // TMEM score buffers
+constexpr int kTcTmemCols = 512;               // S buffers at columns 0, 64, 128, 192; O of group g at 256 + 64 g
+constexpr int kTcOCol = kSBufs * kTcRows;
 // Named barriers: 1 + g for softmax group g, kBarSoft for both groups, kBarTmem for warps 1-9.
 constexpr int kBarSoft = 3, kBarTmem = 4;
 
 // Shared-memory layout, from a 1024-byte aligned base.
-constexpr int kOffRing = 0;
-constexpr int kOffQ = kOffRing + kTcStages * kTcStage;
+constexpr int kOffK = 0;
+constexpr int kOffV = kOffK + kKStages * kTcHalfTile;
+constexpr int kOffQ = kOffV + kVStages * kTcHalfTile;
 constexpr int kOffP = kOffQ + kTcQBytes;
 constexpr int kOffStats = kOffP + 2 * kTcPBytes;           // per group: max [2][64], sum [2][64], alpha [2][64] (floats)
 constexpr int kOffFlags = kOffStats + 6 * kTcMaxCols * 4;  // int[16]
 constexpr int kOffBars = kOffFlags + 16 * 4;               // uint64 barriers
-// full[S], empty[S], s_full[2], p_full[2], o_done[2], q_full, fin
-constexpr int kNumBars = 2 * kTcStages + 8;
+// k_full[K], k_empty[K], v_full[V], v_empty[V], s_full[4], p_full[2], o_done[2], q_full, fin
+constexpr int kNumBars = 2 * kKStages + 2 * kVStages + kSBufs + 6;
 constexpr int kOffTmem = kOffBars + kNumBars * 8;
 constexpr int kOffTable = (kOffTmem + 16 + 15) / 16 * 16;
 constexpr int kTcAlign = 1024;
@@ -84,9 +95,12 @@ constexpr int kFlagVote = 0;      // [2][4] per-warp rescale votes of each softm
 constexpr int kFlagAbort = 8;     // a bounded wait ran out
 constexpr int kFlagOk = 9;        // [2] result of a group leader's wait, for its group (10: group 1)
 constexpr int kFlagSegOk = 11;    // no wait ran out before a segment's end (for both groups)
-constexpr int kFlagIssued = 12;   // tiles the TMA lane issued
-constexpr int kFlagConsumed = 13;  // tiles whose copies the MMA lane saw land
+constexpr int kFlagKIssued = 12;  // K tiles the TMA lane issued
+constexpr int kFlagVIssued = 13;  // V tiles the TMA lane issued
 constexpr int kFlagMmaLast = 14;  // the MMA lane issued products (fin must be awaited before freeing TMEM)
+
+// Device status bits (include/dkv.h).
+constexpr int kDevTmaTimeout = 0x2, kDevMergeTimeout = 0x4;
 
 // ------------------------------------------------------------ tcgen05 wrappers
 // Shared-memory matrix descriptor: start address, leading and stride byte
@@ -180,9 +194,14 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
     return d;
 }
 
+// Bounded wait by one thread; true when the phase completed.
+__device__ __forceinline__ bool wait_phase(uint64_t* bar, uint32_t parity) { return mbar_wait(smem_u32(bar), parity); }
+// One poll.
+__device__ __forceinline__ bool test_phase(uint64_t* bar, uint32_t parity) { return mbar_try_wait(smem_u32(bar), parity); }
+
 // ------------------------------------------------------------ tiles
-// The CTA's tiles, slab segment by slab segment: a segment is the part of one
-// slab inside the CTA's range [A, B); tiles are 64 rows from the segment's start.
+// The CTA's tiles, slab segment by slab segment; tiles are 64 rows from the
+// segment's start.
 struct TileWalk {
     Cursor cu;
     int hend, A, B;
@@ -220,8 +239,19 @@ __device__ void load_q_tc(const DecodeArgs& a, int h, unsigned char* sQ, int tid
     }
 }
 
-// Bounded wait by one lane; true when the phase completed.
-__device__ __forceinline__ bool wait_phase(uint64_t* bar, uint32_t parity) { return mbar_wait(smem_u32(bar), parity); }
+// Idle polling of the TMA and MMA lanes is bounded like every wait: kWaitSpins
+// polls without progress or kWaitNs of globaltimer.
+struct IdleBound {
+    int spins = 0;
+    unsigned long long t0 = 0;
+    __device__ void progress() { spins = 0; }
+    __device__ bool expired()
+    {
+        if (spins == 0) t0 = global_ns();
+        ++spins;
+        return spins >= kWaitSpins || ((spins & 63) == 0 && global_ns() - t0 > kWaitNs);
+    }
+};
 
 template <int G>
 __global__ void __launch_bounds__(kTcThreads, 1)
@@ -229,7 +259,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 {
     extern __shared__ __align__(128) unsigned char smem_raw[];
     unsigned char* sm = smem_raw + ((kTcAlign - (smem_u32(smem_raw) & (kTcAlign - 1))) & (kTcAlign - 1));
-    unsigned char* ring = sm + kOffRing;
+    unsigned char* ringK = sm + kOffK;
+    unsigned char* ringV = sm + kOffV;
     unsigned char* sQ = sm + kOffQ;
     unsigned char* sP = sm + kOffP;
     float* g_max = reinterpret_cast<float*>(sm + kOffStats);  // [2][64] running max of each group, at a segment's end
@@ -237,13 +268,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     float* g_alpha = g_sum + 2 * kTcMaxCols;                   // [2][64] rescale factors of a tile
     volatile int* flags = reinterpret_cast<volatile int*>(sm + kOffFlags);
     uint64_t* bars = reinterpret_cast<uint64_t*>(sm + kOffBars);
-    uint64_t* full = bars;                    // [S] the stage's copies landed
-    uint64_t* empty = bars + kTcStages;       // [S] the stage's products are done
-    uint64_t* s_full = bars + 2 * kTcStages;  // [2] S of tile t (buffer t & 1) is done
-    uint64_t* p_full = s_full + 2;            // [2] P of tile t is written
-    uint64_t* o_done = p_full + 2;            // [2] the O product of tile t is done
-    uint64_t* q_full = o_done + 2;            // the segment's Q is in place
-    uint64_t* fin = q_full + 1;               // drain after a timeout
+    uint64_t* k_full = bars;                        // [K] the stage's K rows landed
+    uint64_t* k_empty = k_full + kKStages;          // [K] its score product is done
+    uint64_t* v_full = k_empty + kKStages;          // [V] the stage's V rows landed
+    uint64_t* v_empty = v_full + kVStages;          // [V] its output product is done
+    uint64_t* s_full = v_empty + kVStages;          // [4] S of tile t (buffer t % 4) is done
+    uint64_t* p_full = s_full + kSBufs;             // [2] P of tile t (buffer t % 2) is written
+    uint64_t* o_done = p_full + 2;                  // [2] the output product of tile t is done
+    uint64_t* q_full = o_done + 2;                  // the segment's Q is in place
+    uint64_t* fin = q_full + 1;                     // drain after a timeout
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + kOffTmem);
     const SeqTable tab = seq_table_at(sm + kOffTable, a);
 
@@ -256,9 +289,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     else
         load_slab_cache(a, tab, 32, kTcThreads - 32);
     if (tid == 32) {
-        for (int i = 0; i < 2 * kTcStages + 6; ++i) mbar_init(smem_u32(&bars[i]), 1);
-        mbar_init(smem_u32(q_full), 1);
-        mbar_init(smem_u32(fin), 1);
+        for (int i = 0; i < kNumBars; ++i) mbar_init(smem_u32(&bars[i]), 1);
         for (int i = 0; i < 16; ++i) flags[i] = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         fence_proxy_async_smem();
@@ -268,9 +299,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
     const int R = slab_start(a, tab, NHl);
     if (c == 0 && warp == 2) {
-        // Slab bounds for the combine launch (after the wait: the previous kernel may read them).
+        // Slabs with no rows belong to no CTA: their outputs are zero (after the
+        // wait, as every write of out).
         pdl_wait();
-        for (int h = lane; h <= NHl; h += 32) a.tc_bounds[h] = slab_start(a, tab, h);
+        for (int h = 0; h < NHl; ++h)
+            if (slab_start(a, tab, h) == slab_start(a, tab, h + 1))
+                for (int j = 0; j < a.NC; ++j)
+                    write_out<G>(a, h / a.Hkv, h % a.Hkv, j, make_float4(0.f, 0.f, 0.f, 0.f), 0.f, lane);
     }
     const int A = part_start(c, R, a.nctas), Bc = part_start(c + 1, R, a.nctas);
     if (A >= Bc) return;  // uniform: this CTA has no rows (no TMEM taken yet)
@@ -283,31 +318,52 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
     if (warp == 0) {
         // ---------------------------------------------------------------- TMA
-        // Starts at once: the copies need no TMEM.
+        // Starts at once (the copies need no TMEM); K and V of a tile go to their
+        // own rings, each issued as soon as its stage is free.
         if (lane == 0) {
             const uint64_t pol = evict_first_policy();
-            TileWalk w;
-            w.begin(a, tab, hfirst, hend, A, Bc);
-            int t = 0;
-            for (; w.more(); ++t, w.next(a, tab)) {
-                if (flags[kFlagAbort]) break;
-                const int s = t % kTcStages;
-                if (t >= kTcStages && !wait_phase(&empty[s], ((t / kTcStages) - 1) & 1)) {
-                    atomicOr(a.status, 0x2 /* DKV_DEV_TMA_TIMEOUT */);
+            TileWalk wk, wv;
+            wk.begin(a, tab, hfirst, hend, A, Bc);
+            wv = wk;
+            int tk = 0, tv = 0;
+            bool waited = false;
+            IdleBound idle;
+            while ((wk.more() || wv.more()) && !flags[kFlagAbort]) {
+                bool moved = false;
+                if (wk.more() && (tk < kKStages || test_phase(&k_empty[tk % kKStages], ((tk / kKStages) - 1) & 1))) {
+                    if (tk == PRE && !waited) {
+                        pdl_wait();  // later copies after the previous kernel, as in the other kernels
+                        waited = true;
+                    }
+                    const int s = tk % kKStages, row = wk.cache_row();
+                    const uint32_t bar = smem_u32(&k_full[s]), dst = smem_u32(ringK + s * kTcHalfTile);
+                    mbar_arrive_expect_tx(bar, kTcHalfTile);
+                    tma_box(dst, &maps.k, 0, row, bar, pol);
+                    tma_box(dst + kTcBox, &maps.k, 64, row, bar, pol);
+                    ++tk;
+                    wk.next(a, tab);
+                    moved = true;
+                }
+                if (wv.more() && tv < tk && (tv < kVStages || test_phase(&v_empty[tv % kVStages], ((tv / kVStages) - 1) & 1))) {
+                    const int s = tv % kVStages, row = wv.cache_row();
+                    const uint32_t bar = smem_u32(&v_full[s]), dst = smem_u32(ringV + s * kTcHalfTile);
+                    mbar_arrive_expect_tx(bar, kTcHalfTile);
+                    tma_box(dst, &maps.v, 0, row, bar, pol);
+                    tma_box(dst + kTcBox, &maps.v, 64, row, bar, pol);
+                    ++tv;
+                    wv.next(a, tab);
+                    moved = true;
+                }
+                if (moved) {
+                    idle.progress();
+                } else if (idle.expired()) {
+                    atomicOr(a.status, kDevTmaTimeout);
                     flags[kFlagAbort] = 1;
                     break;
                 }
-                if (t == PRE) pdl_wait();  // later copies after the previous kernel, as in the other kernels
-                const int row = w.cache_row();
-                const uint32_t bar = smem_u32(&full[s]);
-                const uint32_t dst = smem_u32(ring + s * kTcStage);
-                mbar_arrive_expect_tx(bar, kTcStage);
-                tma_box(dst, &maps.k, 0, row, bar, pol);
-                tma_box(dst + kTcBox, &maps.k, 64, row, bar, pol);
-                tma_box(dst + 2 * kTcBox, &maps.v, 0, row, bar, pol);
-                tma_box(dst + 3 * kTcBox, &maps.v, 64, row, bar, pol);
             }
-            flags[kFlagIssued] = t;
+            flags[kFlagKIssued] = tk;
+            flags[kFlagVIssued] = tv;
         }
     } else {
         if (warp == 1) {
@@ -323,81 +379,89 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
     if (warp == 1) {
         // ---------------------------------------------------------------- MMA
+        // Score products run up to kSBufs tiles ahead of the output products; a
+        // score product needs its K stage, its S buffer free (the output product
+        // of tile t - 4 issued, so its softmax is done) and, first in a segment,
+        // the segment's Q; an output product needs its P and its V stage.
         if (lane == 0) {
             const uint32_t id1 = idesc(kTcQRows, kTcRows, 0, 0);
             const uint32_t id2 = idesc(128, NCpad, 1, 0);
-            TileWalk w;
-            w.begin(a, tab, hfirst, hend, A, Bc);
-            int t = 0, seg = 0, seg_start = 0, prev_seg_start = 0;
-            bool issued = false, ok = true;
-            // O^T += V^T P for tile u into its group's accumulator (u & 1), then
-            // release the stage. A group's first tile of a segment starts it afresh.
-            auto mma2 = [&](int u, int u_seg_start) -> bool {
-                const int b = u & 1, s = u % kTcStages;
-                if (!wait_phase(&p_full[b], (u >> 1) & 1)) return false;
-                tc_fence_after();
-                const uint32_t v0 = smem_u32(ring + s * kTcStage + 2 * kTcBox);
-                const uint32_t p0 = smem_u32(sP + b * kTcPBytes);
-                const uint32_t o = tmem + kTcOCol + b * kTcMaxCols;
-                const uint32_t fresh = (u - u_seg_start) < 2;
-#pragma unroll
-                for (int k = 0; k < kTcRows / 16; ++k) {
-                    const uint64_t av = sdesc(v0 + k * 2048, kTcBox, 1024);
-                    umma(o, av, sdesc(p0 + k * 32, 16, 1024), id2, (fresh && k == 0) ? 0u : 1u);
-                    umma(o, av, sdesc(p0 + kTcMaxCols * 128 + k * 32, 16, 1024), id2, 1u);
-                }
-                umma_commit(smem_u32(&o_done[b]));
-                umma_commit(smem_u32(&empty[s]));
-                return true;
-            };
-            for (; w.more(); ++t, w.next(a, tab)) {
+            TileWalk w1;
+            w1.begin(a, tab, hfirst, hend, A, Bc);
+            int t1 = 0, t2 = 0, seg = 0, seg_start = 0;
+            // Segment start of tiles between the two products (at most kSBufs).
+            int starts[kSBufs] = {0, 0, 0, 0};
+            bool issued = false, ok = true, qseen = false;
+            IdleBound idle;
+            while ((w1.more() || t2 < t1) && ok) {
                 if (flags[kFlagAbort]) {
                     ok = false;
                     break;
                 }
-                const int s = t % kTcStages, b = t & 1;
-                const bool first = w.first();
-                if (!wait_phase(&full[s], (t / kTcStages) & 1)) {
-                    ok = false;
-                    break;
-                }
-                flags[kFlagConsumed] = t + 1;
-                if (first) {
-                    if (!wait_phase(q_full, seg++ & 1)) {
-                        ok = false;
-                        break;
+                bool moved = false;
+                if (w1.more() && t1 < t2 + kSBufs) {
+                    const int s = t1 % kKStages;
+                    const bool first = w1.first();
+                    if (first && !qseen && test_phase(q_full, seg & 1)) {
+                        ++seg;
+                        seg_start = t1;
+                        qseen = true;  // this segment's Q is in place
                     }
-                    prev_seg_start = seg_start;
-                    seg_start = t;
-                }
-                tc_fence_after();
-                // S^T[64 x 64] = Q[64 x 128] K^T: k-steps of 16 dims (+32 B inside a 64-dim half).
-                const uint32_t q0 = smem_u32(sQ), k0 = smem_u32(ring + s * kTcStage);
+                    if ((!first || qseen) && test_phase(&k_full[s], (t1 / kKStages) & 1)) {
+                        tc_fence_after();
+                        // S^T[64 x 64] = Q[64 x 128] K^T: k-steps of 16 dims (+32 B inside a 64-dim half).
+                        const uint32_t q0 = smem_u32(sQ), k0 = smem_u32(ringK + s * kTcHalfTile);
+                        const uint32_t d = tmem + (t1 % kSBufs) * kTcRows;
 #pragma unroll
-                for (int k = 0; k < 8; ++k)
-                    umma(tmem + kTcSCol + b * kTcRows, sdesc(q0 + (k >> 2) * kTcQHalf + (k & 3) * 32, 16, 1024),
-                         sdesc(k0 + (k >> 2) * kTcBox + (k & 3) * 32, 16, 1024), id1, k > 0 ? 1u : 0u);
-                umma_commit(smem_u32(&s_full[b]));
-                issued = true;
-                if (t > 0 && !mma2(t - 1, first ? prev_seg_start : seg_start)) {
+                        for (int k = 0; k < 8; ++k)
+                            umma(d, sdesc(q0 + (k >> 2) * kTcQHalf + (k & 3) * 32, 16, 1024),
+                                 sdesc(k0 + (k >> 2) * kTcBox + (k & 3) * 32, 16, 1024), id1, k > 0 ? 1u : 0u);
+                        umma_commit(smem_u32(&s_full[t1 % kSBufs]));
+                        umma_commit(smem_u32(&k_empty[s]));
+                        starts[t1 % kSBufs] = seg_start;
+                        issued = true;
+                        qseen = false;
+                        ++t1;
+                        w1.next(a, tab);
+                        moved = true;
+                    }
+                }
+                if (t2 < t1) {
+                    const int b = t2 & 1, s = t2 % kVStages;
+                    if (test_phase(&p_full[b], (t2 >> 1) & 1) && test_phase(&v_full[s], (t2 / kVStages) & 1)) {
+                        tc_fence_after();
+                        // O^T += V^T P into the group's accumulator; a group's first tile of
+                        // a segment starts it afresh.
+                        const uint32_t v0 = smem_u32(ringV + s * kTcHalfTile);
+                        const uint32_t p0 = smem_u32(sP + b * kTcPBytes);
+                        const uint32_t o = tmem + kTcOCol + b * kTcMaxCols;
+                        const uint32_t fresh = (t2 - starts[t2 % kSBufs]) < 2;
+#pragma unroll
+                        for (int k = 0; k < kTcRows / 16; ++k) {
+                            const uint64_t av = sdesc(v0 + k * 2048, kTcBox, 1024);
+                            umma(o, av, sdesc(p0 + k * 32, 16, 1024), id2, (fresh && k == 0) ? 0u : 1u);
+                            umma(o, av, sdesc(p0 + kTcMaxCols * 128 + k * 32, 16, 1024), id2, 1u);
+                        }
+                        umma_commit(smem_u32(&o_done[b]));
+                        umma_commit(smem_u32(&v_empty[s]));
+                        ++t2;
+                        moved = true;
+                    }
+                }
+                if (moved) {
+                    idle.progress();
+                } else if (idle.expired()) {
                     ok = false;
-                    break;
                 }
             }
-            if (ok && t > 0 && !mma2(t - 1, seg_start)) ok = false;
             if (!ok) {
-                atomicOr(a.status, 0x2 /* DKV_DEV_TMA_TIMEOUT */);
+                atomicOr(a.status, kDevTmaTimeout);
                 flags[kFlagAbort] = 1;
             }
             flags[kFlagMmaLast] = issued ? 1 : 0;
         }
     } else if (warp >= 2) {
         // ---------------------------------------------------------------- softmax groups and epilogue
-        // Group gi takes the tiles t with t % 2 == gi, with its own running max and
-        // sum of each column and its own O accumulator; the two are merged at the
-        // end of a segment. Thread (quarter, lane < 16) owns column 16 quarter + lane
-        // (TMEM lane 32 quarter + lane of S^T, all 64 rows of a tile); for O, thread
-        // (quarter, lane) owns dimension 32 quarter + lane.
         const int gi = (warp - 2) >> 2;
         const int quarter = warp & 3;
         const int gt = tid - 64 - kTcGroup * gi;   // 0..127 within the group
@@ -431,17 +495,19 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             }
             const bool last = w.last();
             if ((t & 1) == gi) {
-                const int b = gi, s = t % kTcStages;
+                const int b = gi;
                 const int cnt = w.cnt();
                 const bool gfirst = t - seg_start < 2;  // the group's first tile of the segment
                 last_mine = t;
-                // The tile's scores, and the end of the group's previous O product
-                // (it read P buffer b, and rescaling O needs it done).
+                // The tile's scores; the end of the group's previous output product (it
+                // read P buffer b, and rescaling O needs it done); for a partial tile,
+                // its V rows (zeroed below).
                 if (gleader) {
-                    bool ok = !flags[kFlagAbort] && wait_phase(&s_full[b], (t >> 1) & 1);
+                    bool ok = !flags[kFlagAbort] && wait_phase(&s_full[t % kSBufs], (t / kSBufs) & 1);
                     if (ok && t >= 2) ok = wait_phase(&o_done[b], ((t - 2) >> 1) & 1);
-                    if (!ok) {
-                        atomicOr(a.status, 0x2 /* DKV_DEV_TMA_TIMEOUT */);
+                    if (ok && cnt < kTcRows) ok = wait_phase(&v_full[t % kVStages], (t / kVStages) & 1);
+                    if (!ok && !flags[kFlagAbort]) {
+                        atomicOr(a.status, kDevTmaTimeout);
                         flags[kFlagAbort] = 1;
                     }
                     flags[kFlagOk + gi] = ok;
@@ -453,8 +519,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 } else {
                     tc_fence_after();
                     float sc[kTcRows];
-                    tmem_ld32(tmem + lane_addr + kTcSCol + b * kTcRows, *reinterpret_cast<float(*)[32]>(sc));
-                    tmem_ld32(tmem + lane_addr + kTcSCol + b * kTcRows + 32, *reinterpret_cast<float(*)[32]>(sc + 32));
+                    const uint32_t sb = tmem + lane_addr + (t % kSBufs) * kTcRows;
+                    tmem_ld32(sb, *reinterpret_cast<float(*)[32]>(sc));
+                    tmem_ld32(sb + 32, *reinterpret_cast<float(*)[32]>(sc + 32));
                     if (cnt < kTcRows) {
 #pragma unroll
                         for (int i = 0; i < kTcRows; ++i)
@@ -521,7 +588,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     }
                     if (cnt < kTcRows) {
                         // V rows past the segment: zeros (their p is 0, but 0 * inf or 0 * nan would not be).
-                        unsigned char* v0 = ring + s * kTcStage + 2 * kTcBox;
+                        unsigned char* v0 = ringV + (t % kVStages) * kTcHalfTile;
                         for (int i = gt; i < (kTcRows - cnt) * 16; i += kTcGroup) {
                             const int r = cnt + (i >> 4), k = i & 15;
                             *reinterpret_cast<uint4*>(v0 + (k >> 3) * kTcBox + r * 128 + ((k & 7) << 4)) =
@@ -537,7 +604,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             if (!last) continue;
 
             // ---- end of a segment, both groups: the next segment's Q, then the merge of
-            // the two groups' states and this segment's output or partial.
+            // the two groups' states, and this segment's output or partial.
             if (leader) flags[kFlagSegOk] = !flags[kFlagAbort];
             named_sync(kBarSoft, kTcSoft);  // every S product of the segment was seen done by its group
             const bool seg_ok = flags[kFlagSegOk];
@@ -560,15 +627,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 g_sum[gi * kTcMaxCols + col] = l;
             }
             named_sync(kBarSoft, kTcSoft);
-            // The next segment's Q is in place: its first S product may start. (It must be
-            // released before the waits below: the MMA lane issues this segment's last O
-            // product only after that S product.)
+            // The next segment's Q is in place: its score products may start.
             if (leader && has_next) mbar_arrive(smem_u32(q_full));
             if (gleader) {
                 bool ok = seg_ok;
                 if (ok && last_mine >= 0) ok = wait_phase(&o_done[gi], (last_mine >> 1) & 1);
                 if (seg_ok && !ok) {
-                    atomicOr(a.status, 0x2 /* DKV_DEV_TMA_TIMEOUT */);
+                    atomicOr(a.status, kDevTmaTimeout);
                     flags[kFlagAbort] = 1;
                 }
                 flags[kFlagOk + gi] = ok;
@@ -578,7 +643,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             const bool merge_ok = flags[kFlagOk] && flags[kFlagOk + 1];
             stop = !merge_ok;
             tc_fence_after();
-            // Merge: group gi writes the columns 32 gi .. 32 gi + 31 of every dimension.
+            // Merge of the groups: group gi writes the columns 32 gi .. 32 gi + 31 of every dimension.
             const int oc0 = 32 * gi;
             const int bq = h / a.Hkv, g = h - bq * a.Hkv;
             const int64_t slot = (int64_t)c + h;
@@ -603,8 +668,96 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     }
                 }
             }
+            if (merge_ok && !whole) __threadfence();  // the partial, before the count below
             // g_max / g_sum are rewritten at the next segment's end, after these reads.
             named_sync(kBarSoft, kTcSoft);
+            if (merge_ok && !whole && leader) {
+                // This CTA's partial of slab h is written: count it in.
+                __threadfence();
+                atomicAdd(a.slab_count + (int64_t)h * kMaxCols * 2, 1);
+            }
+        }
+
+        // ---- the CTA's share of the merges of its slabs that span several CTAs
+        // (its first and its last segment; the slabs in between were whole).
+        const int P = a.nctas;
+        for (int e = 0; e < 2; ++e) {
+            const int h = e == 0 ? hfirst : hend - 1;
+            if (e == 1 && h == hfirst) break;
+            const int p0 = slab_start(a, tab, h), p1 = slab_start(a, tab, h + 1);
+            int c0 = 0, c1 = 0;
+            const int nct = ctas_of_slab(p0, p1, R, P, &c0, &c1);
+            if (nct <= 1) continue;  // uniform: written at its segment's end
+            int32_t* ctr = a.slab_count + (int64_t)h * kMaxCols * 2;
+            if (leader) {
+                // Every CTA of the slab counts in once its partial is written; the CTAs
+                // are all resident (cooperative launch), so the count completes.
+                bool ok = !flags[kFlagAbort];
+                if (ok) {
+                    ok = false;
+                    const unsigned long long t0 = global_ns();
+                    for (int i = 1; i < kWaitSpins; ++i) {
+                        int n;
+                        asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(n) : "l"(ctr) : "memory");
+                        if (n >= nct + a.merge_extra) {
+                            ok = true;
+                            break;
+                        }
+                        if ((i & 63) == 0 && global_ns() - t0 > kWaitNs) break;
+                    }
+                    if (!ok) atomicOr(a.status, kDevMergeTimeout);
+                }
+                flags[kFlagSegOk] = ok;
+            }
+            named_sync(kBarSoft, kTcSoft);
+            if (flags[kFlagSegOk]) {
+                // Rank of this CTA among the slab's CTAs (every CTA of the range is live
+                // when the layer has at least one row per CTA).
+                const bool all_live = R >= P;
+                int k = 0;
+                if (all_live) {
+                    k = c - c0;
+                } else {
+                    for (int cc = c0; cc < c; ++cc) k += part_start(cc, R, P) < part_start(cc + 1, R, P) ? 1 : 0;
+                }
+                const int j0 = (int)((int64_t)k * NC / nct), j1 = (int)((int64_t)(k + 1) * NC / nct);
+                const int hb = h / a.Hkv, hg = h - hb * a.Hkv;
+                // Columns j0 .. j1-1: warp (gi, quarter) takes j0 + 4 gi + quarter, then
+                // every 8th; a lane covers 4 dims.
+                for (int j = j0 + 4 * gi + quarter; j < j1; j += 8) {
+                    float M = -INFINITY;
+                    for (int cc = c0; cc <= c1; ++cc)
+                        if (all_live || part_start(cc, R, P) < part_start(cc + 1, R, P))
+                            M = fmaxf(M, __ldcg(a.work_ml + (((int64_t)cc + h) * NC + j) * 2));
+                    float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
+                    float L = 0.f;
+#pragma unroll 4
+                    for (int cc = c0; cc <= c1; ++cc) {
+                        if (!(all_live || part_start(cc, R, P) < part_start(cc + 1, R, P))) continue;
+                        const int64_t sj = ((int64_t)cc + h) * NC + j;
+                        const float2 ml = __ldcg(reinterpret_cast<const float2*>(a.work_ml + sj * 2));
+                        const float f = (ml.x == -INFINITY) ? 0.f : ex2(ml.x - M);
+                        L = fmaf(ml.y, f, L);
+                        const float4 v = __ldcg(reinterpret_cast<const float4*>(a.work_o + sj * kHeadDim) + lane);
+                        O.x = fmaf(v.x, f, O.x);
+                        O.y = fmaf(v.y, f, O.y);
+                        O.z = fmaf(v.z, f, O.z);
+                        O.w = fmaf(v.w, f, O.w);
+                    }
+                    write_out<G>(a, hb, hg, j, O, L, lane);
+                }
+            }
+            named_sync(kBarSoft, kTcSoft);
+            if (leader) {
+                // The last CTA of the slab to finish its share resets the counters for
+                // the next call (every wait on the arrival count is over by then).
+                const int done = atomicAdd(ctr + 1, 1);
+                if (done == nct - 1) {
+                    ctr[0] = 0;
+                    ctr[1] = 0;
+                    __threadfence();
+                }
+            }
         }
     }
 
@@ -612,11 +765,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     tc_fence_before();
     __syncthreads();
     if (flags[kFlagAbort]) {
-        // Drain what is still in flight, with the same bound, before the CTA exits.
+        // Drain what is still in flight, with the same bound, before the CTA exits:
+        // the copies of every stage issued (a landed stage's wait returns at once),
+        // and the products (a final commit).
         if (tid == 0) {
-            const int issued = flags[kFlagIssued], consumed = flags[kFlagConsumed];
-            for (int u = max(consumed, issued - kTcStages); u < issued; ++u)
-                wait_phase(&full[u % kTcStages], (u / kTcStages) & 1);
+            const int nk = flags[kFlagKIssued], nv = flags[kFlagVIssued];
+            for (int u = max(0, nk - kKStages); u < nk; ++u) wait_phase(&k_full[u % kKStages], (u / kKStages) & 1);
+            for (int u = max(0, nv - kVStages); u < nv; ++u) wait_phase(&v_full[u % kVStages], (u / kVStages) & 1);
         }
         if (tid == 32 && flags[kFlagMmaLast]) {
             umma_commit(smem_u32(fin));
@@ -628,48 +783,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     tc_fence_after();
     if (warp == 1)
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTcTmemCols));
-}
-
-// Merge of the CTA partials of slab h, column j (one CTA of 128 threads, thread d
-// = dimension d): slabs wholly inside one CTA were written by the decode kernel;
-// slabs with no rows get zeros.
-template <int G>
-__global__ void __launch_bounds__(128) decode_tc_combine_kernel(const DecodeArgs a)
-{
-    pdl_launch_dependents();
-    pdl_wait();
-    const int NC = a.NC;
-    const int h = blockIdx.x / NC, j = blockIdx.x - h * NC;
-    const int NHl = a.B * a.Hkv;
-    const int R = a.tc_bounds[NHl];
-    const int p0 = a.tc_bounds[h], p1 = a.tc_bounds[h + 1];
-    const int b = h / a.Hkv, g = h - b * a.Hkv;
-    float* dst = a.out + out_row<G>(a, b, g, j) * kHeadDim;
-    const int d = threadIdx.x;
-    if (p1 <= p0) {
-        dst[d] = 0.f;
-        return;
-    }
-    const int P = a.nctas;
-    int c0 = 0, c1 = 0;
-    const int nct = ctas_of_slab(p0, p1, R, P, &c0, &c1);
-    if (nct <= 1) return;
-    const bool all_live = R >= P;
-    float M = -INFINITY;
-    for (int cc = c0; cc <= c1; ++cc)
-        if (all_live || part_start(cc, R, P) < part_start(cc + 1, R, P))
-            M = fmaxf(M, __ldcg(a.work_ml + (((int64_t)cc + h) * NC + j) * 2));
-    float O = 0.f, Ls = 0.f;
-#pragma unroll 4
-    for (int cc = c0; cc <= c1; ++cc) {
-        if (!(all_live || part_start(cc, R, P) < part_start(cc + 1, R, P))) continue;
-        const int64_t sj = ((int64_t)cc + h) * NC + j;
-        const float2 ml = __ldcg(reinterpret_cast<const float2*>(a.work_ml + sj * 2));
-        const float f = (ml.x == -INFINITY) ? 0.f : ex2(ml.x - M);
-        Ls = fmaf(ml.y, f, Ls);
-        O = fmaf(__ldcg(a.work_o + sj * kHeadDim + d), f, O);
-    }
-    dst[d] = Ls > 0.f ? O / Ls : 0.f;
 }
 
 template <int G>
@@ -685,7 +798,7 @@ cudaError_t config_tc_g(int B, DecodeConfig* cfg)
         cudaSuccess)
         return e;
     if (per_sm < 1) return cudaErrorInvalidConfiguration;
-    cfg->nctas = sms;  // one CTA per SM: the TMEM allocation never waits for another CTA's
+    cfg->nctas = sms;  // one CTA per SM: co-resident (cooperative), and the TMEM allocation never waits
     cfg->nwarps = kTcThreads / 32;
     cfg->smem_bytes = smem;
     return cudaSuccess;
@@ -695,11 +808,23 @@ template <int G>
 cudaError_t launch_tc_g(const DecodeArgs& a, const CacheMaps& maps, const DecodeConfig& cfg, cudaStream_t st)
 {
     if (cfg.nwarps != kTcThreads / 32 || cfg.smem_bytes < tc_smem_bytes(a.B) || a.nctas < 1 || a.nctas > cfg.nctas ||
-        a.NC < 1 || a.NC > kTcMaxCols || !a.tc_bounds)
+        a.NC < 1 || a.NC > kTcMaxCols || !a.slab_count)
         return cudaErrorInvalidConfiguration;
-    cudaError_t e = launch_pdl(decode_tc_kernel<G>, a.nctas, kTcThreads, cfg.smem_bytes, st, a, maps);
-    if (e != cudaSuccess) return e;
-    return launch_pdl(decode_tc_combine_kernel<G>, a.B * a.Hkv * a.NC, 128, 0, st, a);
+    // Cooperative (every CTA resident: a CTA waits for the other CTAs of its slabs)
+    // and programmatic stream serialization, as the other decode kernels.
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = dim3(a.nctas);
+    lc.blockDim = dim3(kTcThreads);
+    lc.dynamicSmemBytes = cfg.smem_bytes;
+    lc.stream = st;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[1].id = cudaLaunchAttributeCooperative;
+    attr[1].val.cooperative = 1;
+    lc.attrs = attr;
+    lc.numAttrs = 2;
+    return cudaLaunchKernelEx(&lc, decode_tc_kernel<G>, a, maps);
 }
 
 }  // namespace

@@ -82,7 +82,6 @@ struct DecodeArgs {
     int Q;                  // queries per sequence (1 for the decode step); q and out are [B][Q][H][128]
     int NC;                 // columns per slab: Q * G; partial records hold NC rows of 128 + 2 floats
     int merge_extra;        // partials a fused merge waits for beyond the other CTAs' (0; 1 injects a wait that runs out)
-    int32_t* tc_bounds;     // [B*Hkv+1] first layer row of each slab, written by the tcgen05 kernel for its combine
 };
 
 // Most columns (queries x group heads) one decode call handles; the plan's
@@ -99,27 +98,24 @@ struct DecodeConfig {
 
 // Carve-up of the split-K workspace, in floats from its base: the (CTA, slab)
 // partials o [slots][slot_cols][128] and (m, l) [slots][slot_cols][2], the warp
-// records o [warp_records][warp_cols][128] and (m, l) [warp_records][warp_cols][2],
-// and the slab bounds of the tcgen05 kernel's combine, int32 [slabs + 1]. Each
-// region starts on a 256-byte boundary: the kernels move o with 16-byte vector
+// records o [warp_records][warp_cols][128] and (m, l) [warp_records][warp_cols][2].
+// Each region starts on a 256-byte boundary: the kernels move o with 16-byte vector
 // accesses and (m, l) with 8-byte ones, whatever slots x columns is (an odd
 // product would otherwise leave the warp records 8-byte aligned).
 struct WorkspaceLayout {
-    int64_t work_o, work_ml, warp_o, warp_ml, bounds;  // region offsets (floats)
+    int64_t work_o, work_ml, warp_o, warp_ml;  // region offsets (floats)
     int64_t total;                                     // floats of the whole workspace
 };
 constexpr int64_t kWorkAlignFloats = 64;  // 256 bytes
 inline int64_t round_up_work(int64_t n) { return (n + kWorkAlignFloats - 1) / kWorkAlignFloats * kWorkAlignFloats; }
-inline WorkspaceLayout workspace_layout(int64_t slots, int slot_cols, int64_t warp_records, int warp_cols,
-                                        int64_t slabs_per_layer)
+inline WorkspaceLayout workspace_layout(int64_t slots, int slot_cols, int64_t warp_records, int warp_cols)
 {
     WorkspaceLayout w;
     w.work_o = 0;
     w.work_ml = w.work_o + round_up_work(slots * slot_cols * kHeadDim);
     w.warp_o = w.work_ml + round_up_work(slots * slot_cols * 2);
     w.warp_ml = w.warp_o + round_up_work(warp_records * warp_cols * kHeadDim);
-    w.bounds = w.warp_ml + round_up_work(warp_records * warp_cols * 2);
-    w.total = w.bounds + round_up_work(slabs_per_layer + 1);
+    w.total = w.warp_ml + round_up_work(warp_records * warp_cols * 2);
     return w;
 }
 // The workspace of kernels of up to `nctas` CTAs of up to `nwarps` warps
@@ -128,7 +124,7 @@ inline WorkspaceLayout workspace_layout(int64_t slots, int slot_cols, int64_t wa
 // warp of the grid.
 inline WorkspaceLayout decode_workspace(int nctas, int nwarps, int cols, int heads_per_layer)
 {
-    return workspace_layout((int64_t)nctas + heads_per_layer, cols, (int64_t)nctas * nwarps, cols, heads_per_layer);
+    return workspace_layout((int64_t)nctas + heads_per_layer, cols, (int64_t)nctas * nwarps, cols);
 }
 // Grid and shared memory of the partial kernel for group size G on this device.
 cudaError_t decode_config(int G, int B, DecodeConfig* cfg);
@@ -161,7 +157,8 @@ cudaError_t launch_decode_mma_fused(const DecodeArgs& a, const CacheMaps& maps, 
 cudaError_t launch_advance(int32_t* n_app, int B, int reserve, int32_t* status, cudaStream_t st);
 
 // tcgen05 multi-query kernel (dkv_decode_tc.cu): 1 to kTcMaxCols columns, one CTA
-// per SM, followed by its combine launch (one CTA per slab and column).
+// per SM (a cooperative launch), the merge of slabs over several CTAs fused in
+// (uses a.slab_count: entry [h][0][0..1] of each slab).
 cudaError_t decode_config_tc(int G, int B, DecodeConfig* cfg);
 cudaError_t launch_decode_tc(const DecodeArgs& a, const CacheMaps& maps, const DecodeConfig& cfg, cudaStream_t st);
 
