@@ -196,8 +196,21 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
 
 // Bounded wait by one thread; true when the phase completed.
 __device__ __forceinline__ bool wait_phase(uint64_t* bar, uint32_t parity) { return mbar_wait(smem_u32(bar), parity); }
-// One poll.
-__device__ __forceinline__ bool test_phase(uint64_t* bar, uint32_t parity) { return mbar_try_wait(smem_u32(bar), parity); }
+// One poll that never suspends the thread (mbarrier.try_wait may suspend it for a
+// system-defined time while the phase is incomplete, which would stall the
+// schedulers below on one stage while another is ready).
+__device__ __forceinline__ bool test_phase(uint64_t* bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
 
 // ------------------------------------------------------------ tiles
 // The CTA's tiles, slab segment by slab segment; tiles are 64 rows from the
@@ -360,6 +373,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     atomicOr(a.status, kDevTmaTimeout);
                     flags[kFlagAbort] = 1;
                     break;
+                } else {
+                    __nanosleep(32);
                 }
             }
             flags[kFlagKIssued] = tk;
@@ -452,6 +467,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     idle.progress();
                 } else if (idle.expired()) {
                     ok = false;
+                } else {
+                    __nanosleep(20);
                 }
             }
             if (!ok) {
