@@ -11,7 +11,7 @@
 //
 //   warp 0 (one lane)   TMA: a tile's K rows and V rows, each as two 2-D boxes
 //                       (64 rows x 64 dims, 128-byte swizzle), into separate
-//                       rings (4 K stages, 6 V stages): a K stage is released as
+//                       rings (4 K stages, 5 V stages): a K stage is released as
 //                       soon as its score product is done, a V stage only after
 //                       its output product, so V is the deeper ring.
 //   warp 1 (one lane)   MMA: S^T = Q K^T  (M = 64 query-column rows of Q, zero
@@ -26,14 +26,19 @@
 //                       t % 2 == g, with its own running max and sum of every
 //                       column and its own O accumulator (merged at a segment's
 //                       end). With M = 64, row c of S^T (column c) sits in TMEM
-//                       lane 32 (c / 16) + c % 16: thread (quarter, lane < 16)
-//                       owns column 16 quarter + lane, all 64 rows of a tile:
-//                       tile max, lazily rescaled running max (a column's max
+//                       lane 32 (c / 16) + c % 16; a 16x32bx2 TMEM load gives
+//                       lanes l and l + 16 of warp (group, quarter) column
+//                       16 quarter + l, rows 0-31 and 32-63 of the tile: tile
+//                       max (one shuffle joins the halves), lazily rescaled
+//                       running max (a column's max
 //                       moves only when a score tops it by kSlack; O is then
 //                       rescaled in TMEM), P = 2^(s - m) written to shared memory
 //                       as the B operand of the output product, V rows past a
 //                       segment zeroed. For O, thread (quarter, lane) owns
 //                       dimension 32 quarter + lane (TMEM lane).
+//
+// Segments alternate between two Q buffers, each loaded two segments ahead, so
+// the score products run on across a slab boundary.
 //
 // A slab wholly inside one CTA is written out at its segment's end. Otherwise
 // each CTA of the slab writes its partial (m, l, o of every column) and counts
@@ -58,7 +63,7 @@ namespace {
 
 constexpr int kTcRows = 64;                    // cache rows per tile
 constexpr int kKStages = 4;                    // K ring stages
-constexpr int kVStages = 6;                    // V ring stages
+constexpr int kVStages = 5;                    // V ring stages
 constexpr int kTcBox = kTcRows * 128;          // one TMA box: 64 rows x 64 dims of bf16 (8 KB)
 constexpr int kTcHalfTile = 2 * kTcBox;        // K (or V) rows of one tile: dims 0-63, then 64-127
 constexpr int kTcThreads = 320;                // warps: 0 TMA, 1 MMA, 2-5 and 6-9 the two softmax groups
@@ -66,7 +71,7 @@ constexpr int kTcSoft = 256;                   // threads of the softmax warps
 constexpr int kTcGroup = 128;                  // threads of one softmax group
 constexpr int kTcQRows = 64;                   // M of the score product: the most columns
 constexpr int kTcQHalf = kTcQRows * 128;       // one 64-dim half of Q (8 KB)
-constexpr int kTcQBytes = 2 * kTcQHalf;        // Q as the A operand: 64 rows x 128 dims
+constexpr int kTcQBytes = 2 * kTcQHalf;        // Q as the A operand: 64 rows x 128 dims (two buffers: segments alternate)
 constexpr int kTcPBytes = 2 * kTcMaxCols * 128;  // one P buffer: high and low parts, 64 columns x 64 rows each
 constexpr int kSBufs = 4;                      // TMEM score buffers
 constexpr int kTcTmemCols = 512;               // S buffers at columns 0, 64, 128, 192; O of group g at 256 + 64 g
@@ -78,12 +83,12 @@ constexpr int kBarSoft = 3, kBarTmem = 4;
 constexpr int kOffK = 0;
 constexpr int kOffV = kOffK + kKStages * kTcHalfTile;
 constexpr int kOffQ = kOffV + kVStages * kTcHalfTile;
-constexpr int kOffP = kOffQ + kTcQBytes;
+constexpr int kOffP = kOffQ + 2 * kTcQBytes;
 constexpr int kOffStats = kOffP + 2 * kTcPBytes;           // per group: max [2][64], sum [2][64], alpha [2][64] (floats)
 constexpr int kOffFlags = kOffStats + 6 * kTcMaxCols * 4;  // int[16]
 constexpr int kOffBars = kOffFlags + 16 * 4;               // uint64 barriers
-// k_full[K], k_empty[K], v_full[V], v_empty[V], s_full[4], p_full[2], o_done[2], q_full, fin
-constexpr int kNumBars = 2 * kKStages + 2 * kVStages + kSBufs + 6;
+// k_full[K], k_empty[K], v_full[V], v_empty[V], s_full[4], p_full[2], o_done[2], q_full[2], fin
+constexpr int kNumBars = 2 * kKStages + 2 * kVStages + kSBufs + 7;
 constexpr int kOffTmem = kOffBars + kNumBars * 8;
 constexpr int kOffTable = (kOffTmem + 16 + 15) / 16 * 16;
 constexpr int kTcAlign = 1024;
@@ -145,6 +150,24 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32])
     asm volatile(
         "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
         "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// 16 TMEM lanes from taddr: lanes 0-15 of the warp read columns [col, col + 32),
+// lanes 16-31 the same TMEM lanes at columns [col + 32, col + 64).
+__device__ __forceinline__ void tmem_ld16x2(uint32_t taddr, float (&v)[32])
+{
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.16x32bx2.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32], 32;"
         : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
           "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
           "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
@@ -234,6 +257,18 @@ struct TileWalk {
     __device__ void next(const DecodeArgs& a, const SeqTable& t) { cursor_next<kTcRows>(cu, a, t, hend, A, B); }
 };
 
+// Slab of the segment `skip` segments after the one under `cu` (>= hend when
+// there is none).
+__device__ __forceinline__ int later_segment_slab(Cursor cu, const DecodeArgs& a, const SeqTable& t, int hend, int A,
+                                                  int B, int skip)
+{
+    for (int k = 0; k < skip && cu.h < hend; ++k) {
+        ++cu.h;
+        cursor_seek(cu, a, t, hend, A, B);
+    }
+    return cu.h;
+}
+
 // Q of slab h as the A operand: row c (column c: query c / G, head g G + c % G)
 // of 128 bf16 dims, two 64-dim halves, 128-byte swizzle; rows NC.. are zero.
 template <int G>
@@ -288,8 +323,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     uint64_t* s_full = v_empty + kVStages;          // [4] S of tile t (buffer t % 4) is done
     uint64_t* p_full = s_full + kSBufs;             // [2] P of tile t (buffer t % 2) is written
     uint64_t* o_done = p_full + 2;                  // [2] the output product of tile t is done
-    uint64_t* q_full = o_done + 2;                  // the segment's Q is in place
-    uint64_t* fin = q_full + 1;                     // drain after a timeout
+    uint64_t* q_full = o_done + 2;                  // [2] Q buffer b holds the Q of its next segment
+    uint64_t* fin = q_full + 2;                     // drain after a timeout
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + kOffTmem);
     const SeqTable tab = seq_table_at(sm + kOffTable, a);
 
@@ -406,6 +441,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             int t1 = 0, t2 = 0, seg = 0, seg_start = 0;
             // Segment start of tiles between the two products (at most kSBufs).
             int starts[kSBufs] = {0, 0, 0, 0};
+            int qbuf = 0;  // Q buffer of the segment of tile t1
             bool issued = false, ok = true, qseen = false;
             IdleBound idle;
             while ((w1.more() || t2 < t1) && ok) {
@@ -417,7 +453,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 if (w1.more() && t1 < t2 + kSBufs) {
                     const int s = t1 % kKStages;
                     const bool first = w1.first();
-                    if (first && !qseen && test_phase(q_full, seg & 1)) {
+                    if (first && !qseen && test_phase(&q_full[seg & 1], (seg >> 1) & 1)) {
+                        qbuf = seg & 1;
                         ++seg;
                         seg_start = t1;
                         qseen = true;  // this segment's Q is in place
@@ -425,7 +462,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     if ((!first || qseen) && test_phase(&k_full[s], (t1 / kKStages) & 1)) {
                         tc_fence_after();
                         // S^T[64 x 64] = Q[64 x 128] K^T: k-steps of 16 dims (+32 B inside a 64-dim half).
-                        const uint32_t q0 = smem_u32(sQ), k0 = smem_u32(ringK + s * kTcHalfTile);
+                        const uint32_t q0 = smem_u32(sQ + qbuf * kTcQBytes), k0 = smem_u32(ringK + s * kTcHalfTile);
                         const uint32_t d = tmem + (t1 % kSBufs) * kTcRows;
 #pragma unroll
                         for (int k = 0; k < 8; ++k)
@@ -486,17 +523,25 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const bool gleader = gt == 0, leader = st == 0;
         const int gbar = 1 + gi;
         const uint32_t lane_addr = (uint32_t)(32 * quarter) << 16;
-        const int col = 16 * quarter + lane;
-        const bool live = lane < 16 && col < NC;
+        const int half = lane >> 4;                 // rows 32 half .. 32 half + 31 of a tile
+        const int col = 16 * quarter + (lane & 15);
+        const bool live = col < NC;
         const int dim = 32 * quarter + lane;
         const uint32_t my_o = tmem + lane_addr + kTcOCol + gi * kTcMaxCols;
         pdl_wait();  // q and the outputs belong to the previous kernel's epoch
         TileWalk w;
         w.begin(a, tab, hfirst, hend, A, Bc);
+        // Q of the first two segments (buffers 0 and 1).
+        const int h1 = later_segment_slab(w.cu, a, tab, hend, A, Bc, 1);
         load_q_tc<G>(a, w.cu.h, sQ, st);
+        if (h1 < hend) load_q_tc<G>(a, h1, sQ + kTcQBytes, st);
         fence_proxy_async_smem();
         named_sync(kBarSoft, kTcSoft);
-        if (leader) mbar_arrive(smem_u32(q_full));
+        if (leader) {
+            mbar_arrive(smem_u32(&q_full[0]));
+            if (h1 < hend) mbar_arrive(smem_u32(&q_full[1]));
+        }
+        int seg_idx = -1;              // index of the current segment
         float m = -INFINITY, l = 0.f;  // this group's running max (log2 units) and sum of column col
         int t = 0, seg_start = 0;
         int last_mine = -1;            // this group's last tile of the current segment
@@ -506,6 +551,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         for (; w.more() && !stop; ++t, w.next(a, tab)) {
             if (w.first()) {
                 seg_start = t;
+                ++seg_idx;
                 last_mine = -1;
                 m = -INFINITY;
                 l = 0.f;
@@ -535,18 +581,19 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     named_sync(gbar, kTcGroup);  // the flag is rewritten at the group's next tile
                 } else {
                     tc_fence_after();
-                    float sc[kTcRows];
-                    const uint32_t sb = tmem + lane_addr + (t % kSBufs) * kTcRows;
-                    tmem_ld32(sb, *reinterpret_cast<float(*)[32]>(sc));
-                    tmem_ld32(sb + 32, *reinterpret_cast<float(*)[32]>(sc + 32));
+                    float sc[32];  // rows 32 half + i of the tile, column col
+                    tmem_ld16x2(tmem + lane_addr + (t % kSBufs) * kTcRows, sc);
                     if (cnt < kTcRows) {
 #pragma unroll
-                        for (int i = 0; i < kTcRows; ++i)
-                            if (i >= cnt) sc[i] = -INFINITY;  // rows past the segment
+                        for (int i = 0; i < 32; ++i)
+                            if (32 * half + i >= cnt) sc[i] = -INFINITY;  // rows past the segment
                     }
-                    float mt = -INFINITY;
+                    float mx[8];
 #pragma unroll
-                    for (int i = 0; i < kTcRows; ++i) mt = fmaxf(mt, sc[i]);
+                    for (int i = 0; i < 8; ++i) mx[i] = fmaxf(fmaxf(sc[4 * i], sc[4 * i + 1]), fmaxf(sc[4 * i + 2], sc[4 * i + 3]));
+                    float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                                     fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+                    mt = fmaxf(mt, __shfl_xor_sync(kFull, mt, 16));  // the column's other half
                     mt = live ? mt * cs : -INFINITY;  // scale > 0: the max of the scaled scores
                     if (gfirst) {
                         m = mt;
@@ -566,7 +613,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                                 m = mt;
                                 l *= alpha;
                             }
-                            if (lane < 16) g_alpha[gi * kTcMaxCols + col] = alpha;
+                            if (half == 0) g_alpha[gi * kTcMaxCols + col] = alpha;
                             named_sync(gbar, kTcGroup);
                             // The group's O (its previous product is done: waited above).
                             for (int c0 = 0; c0 < NCpad; c0 += 32) {
@@ -581,27 +628,30 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     }
                     // P = 2^(s - m): a bf16 high part (the top 16 bits) and the bf16 of
                     // the remainder, row col of the B operand (64 rows, 128 bytes, swizzled).
-                    if (lane < 16 && col < NCpad) {
-                        const float nm = live ? -m : 0.f;
+                    if (col < NCpad) {
+                        // Columns past NC get p = 0: 2^(s - inf) = 0 for finite or -inf s.
+                        const float nm = live ? -m : -INFINITY;
                         unsigned char* ph = sP + b * kTcPBytes + col * 128;
                         unsigned char* pl = ph + kTcMaxCols * 128;
+                        float ls[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-                        for (int ch = 0; ch < 8; ++ch) {
+                        for (int ch = 0; ch < 4; ++ch) {
                             uint32_t hi[4], lo[4];
 #pragma unroll
                             for (int i = 0; i < 4; ++i) {
-                                const float p0 = live ? ex2(fmaf(sc[8 * ch + 2 * i], cs, nm)) : 0.f;  // 2^-inf = 0
-                                const float p1 = live ? ex2(fmaf(sc[8 * ch + 2 * i + 1], cs, nm)) : 0.f;
-                                l += p0 + p1;
+                                const float p0 = ex2(fmaf(sc[8 * ch + 2 * i], cs, nm));  // 2^-inf = 0
+                                const float p1 = ex2(fmaf(sc[8 * ch + 2 * i + 1], cs, nm));
+                                ls[i] += p0 + p1;
                                 const uint32_t h0 = __float_as_uint(p0) & 0xffff0000u;
                                 const uint32_t h1 = __float_as_uint(p1) & 0xffff0000u;
                                 hi[i] = __byte_perm(h0, h1, 0x7632);
                                 lo[i] = pack_bf16(p0 - __uint_as_float(h0), p1 - __uint_as_float(h1));
                             }
-                            const int off = (ch ^ (col & 7)) << 4;
+                            const int off = ((4 * half + ch) ^ (col & 7)) << 4;
                             *reinterpret_cast<uint4*>(ph + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
                             *reinterpret_cast<uint4*>(pl + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
                         }
+                        l += (ls[0] + ls[1]) + (ls[2] + ls[3]);
                     }
                     if (cnt < kTcRows) {
                         // V rows past the segment: zeros (their p is 0, but 0 * inf or 0 * nan would not be).
@@ -627,25 +677,22 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             const bool seg_ok = flags[kFlagSegOk];
             const int h = w.cu.h, p0h = w.cu.p0, p1h = w.cu.p0 + w.cu.n_h;
             const bool whole = w.cu.s0 == p0h && w.cu.s1 == p1h;
-            bool has_next = false;
-            {
-                TileWalk nx = w;
-                nx.next(a, tab);
-                has_next = nx.more();
-                if (has_next) {
-                    load_q_tc<G>(a, nx.cu.h, sQ, st);
-                    fence_proxy_async_smem();
-                }
+            // Q of the segment after next into this segment's buffer (its score
+            // products are all done: each group saw its tiles' S).
+            const int h2 = later_segment_slab(w.cu, a, tab, hend, A, Bc, 2);
+            if (h2 < hend) {
+                load_q_tc<G>(a, h2, sQ + (seg_idx & 1) * kTcQBytes, st);
+                fence_proxy_async_smem();
             }
             const bool has0 = (t - seg_start >= 1) || ((seg_start & 1) == 0);  // group 0 had a tile here
             const bool has1 = (t - seg_start >= 1) || ((seg_start & 1) == 1);
-            if (lane < 16) {
+            const float lsum = l + __shfl_xor_sync(kFull, l, 16);  // the column's two halves
+            if (half == 0) {
                 g_max[gi * kTcMaxCols + col] = m;
-                g_sum[gi * kTcMaxCols + col] = l;
+                g_sum[gi * kTcMaxCols + col] = lsum;
             }
             named_sync(kBarSoft, kTcSoft);
-            // The next segment's Q is in place: its score products may start.
-            if (leader && has_next) mbar_arrive(smem_u32(q_full));
+            if (leader && h2 < hend) mbar_arrive(smem_u32(&q_full[seg_idx & 1]));
             if (gleader) {
                 bool ok = seg_ok;
                 if (ok && last_mine >= 0) ok = wait_phase(&o_done[gi], (last_mine >> 1) & 1);
@@ -740,27 +787,54 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 const int j0 = (int)((int64_t)k * NC / nct), j1 = (int)((int64_t)(k + 1) * NC / nct);
                 const int hb = h / a.Hkv, hg = h - hb * a.Hkv;
                 // Columns j0 .. j1-1: warp (gi, quarter) takes j0 + 4 gi + quarter, then
-                // every 8th; a lane covers 4 dims.
+                // every 8th. Lane k holds the (m, l) of the slab's k-th CTA partial (32 a
+                // round), so the weights take one round of loads; then each lane covers 4
+                // dims and loads 8 partials' o at a time.
+                const int ncta = c1 - c0 + 1;
                 for (int j = j0 + 4 * gi + quarter; j < j1; j += 8) {
                     float M = -INFINITY;
-                    for (int cc = c0; cc <= c1; ++cc)
-                        if (all_live || part_start(cc, R, P) < part_start(cc + 1, R, P))
+                    for (int k0 = 0; k0 < ncta; k0 += 32) {
+                        const int cc = c0 + k0 + lane;
+                        if (cc <= c1 && (all_live || part_start(cc, R, P) < part_start(cc + 1, R, P)))
                             M = fmaxf(M, __ldcg(a.work_ml + (((int64_t)cc + h) * NC + j) * 2));
-                    float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
+                    }
+#pragma unroll
+                    for (int o = 16; o >= 1; o >>= 1) M = fmaxf(M, __shfl_xor_sync(kFull, M, o));
                     float L = 0.f;
-#pragma unroll 4
-                    for (int cc = c0; cc <= c1; ++cc) {
-                        if (!(all_live || part_start(cc, R, P) < part_start(cc + 1, R, P))) continue;
-                        const int64_t sj = ((int64_t)cc + h) * NC + j;
-                        const float2 ml = __ldcg(reinterpret_cast<const float2*>(a.work_ml + sj * 2));
+                    float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
+                    for (int k0 = 0; k0 < ncta; k0 += 32) {
+                        const int cc = c0 + k0 + lane;
+                        const bool okp = cc <= c1 && (all_live || part_start(cc, R, P) < part_start(cc + 1, R, P));
+                        const float2 ml = okp ? __ldcg(reinterpret_cast<const float2*>(a.work_ml + (((int64_t)cc + h) * NC + j) * 2))
+                                              : make_float2(-INFINITY, 0.f);
                         const float f = (ml.x == -INFINITY) ? 0.f : ex2(ml.x - M);
                         L = fmaf(ml.y, f, L);
-                        const float4 v = __ldcg(reinterpret_cast<const float4*>(a.work_o + sj * kHeadDim) + lane);
-                        O.x = fmaf(v.x, f, O.x);
-                        O.y = fmaf(v.y, f, O.y);
-                        O.z = fmaf(v.z, f, O.z);
-                        O.w = fmaf(v.w, f, O.w);
+                        const int n = min(32, ncta - k0);
+                        for (int u0 = 0; u0 < n; u0 += 8) {
+                            float4 v[8];
+                            float fk[8];
+#pragma unroll
+                            for (int u = 0; u < 8; ++u) {
+                                const int k = u0 + u;
+                                fk[u] = __shfl_sync(kFull, f, k & 31);
+                                const bool okk = __shfl_sync(kFull, okp ? 1 : 0, k & 31) != 0 && k < n;
+                                v[u] = okk ? __ldcg(reinterpret_cast<const float4*>(
+                                                        a.work_o + (((int64_t)c0 + k0 + k + h) * NC + j) * kHeadDim) +
+                                                    lane)
+                                           : make_float4(0.f, 0.f, 0.f, 0.f);
+                                if (!okk) fk[u] = 0.f;
+                            }
+#pragma unroll
+                            for (int u = 0; u < 8; ++u) {
+                                O.x = fmaf(v[u].x, fk[u], O.x);
+                                O.y = fmaf(v[u].y, fk[u], O.y);
+                                O.z = fmaf(v[u].z, fk[u], O.z);
+                                O.w = fmaf(v[u].w, fk[u], O.w);
+                            }
+                        }
                     }
+#pragma unroll
+                    for (int o = 16; o >= 1; o >>= 1) L += __shfl_xor_sync(kFull, L, o);
                     write_out<G>(a, hb, hg, j, O, L, lane);
                 }
             }
