@@ -85,8 +85,8 @@ constexpr int kOffV = kOffK + kKStages * kTcHalfTile;
 constexpr int kOffQ = kOffV + kVStages * kTcHalfTile;
 constexpr int kOffP = kOffQ + 2 * kTcQBytes;
 constexpr int kOffStats = kOffP + 2 * kTcPBytes;           // per group: max [2][64], sum [2][64], alpha [2][64] (floats)
-constexpr int kOffFlags = kOffStats + 6 * kTcMaxCols * 4;  // int[16]
-constexpr int kOffBars = kOffFlags + 16 * 4;               // uint64 barriers
+constexpr int kOffFlags = kOffStats + 6 * kTcMaxCols * 4;  // int[kNumFlags]
+constexpr int kOffBars = kOffFlags + 24 * 4;               // uint64 barriers
 // k_full[K], k_empty[K], v_full[V], v_empty[V], s_full[4], p_full[2], o_done[2], q_full[2], fin
 constexpr int kNumBars = 2 * kKStages + 2 * kVStages + kSBufs + 7;
 constexpr int kOffTmem = kOffBars + kNumBars * 8;
@@ -103,6 +103,13 @@ constexpr int kFlagSegOk = 11;    // no wait ran out before a segment's end (for
 constexpr int kFlagKIssued = 12;  // K tiles the TMA lane issued
 constexpr int kFlagVIssued = 13;  // V tiles the TMA lane issued
 constexpr int kFlagMmaLast = 14;  // the MMA lane issued products (fin must be awaited before freeing TMEM)
+constexpr int kFlagOk2 = 16;      // [2] result of a group leader's second wait of a tile (17: group 1)
+constexpr int kNumFlags = 24;
+
+// Lazy-rescale threshold of the running max (log2 units): P stays below 2^32,
+// far inside fp32 and bf16 range, and a rescale of O in TMEM (a load, multiply
+// and store of every column) is rare even with outlier keys.
+constexpr float kSlackTc = 32.f;
 
 // Device status bits (include/dkv.h).
 constexpr int kDevTmaTimeout = 0x2, kDevMergeTimeout = 0x4;
@@ -338,7 +345,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         load_slab_cache(a, tab, 32, kTcThreads - 32);
     if (tid == 32) {
         for (int i = 0; i < kNumBars; ++i) mbar_init(smem_u32(&bars[i]), 1);
-        for (int i = 0; i < 16; ++i) flags[i] = 0;
+        for (int i = 0; i < kNumFlags; ++i) flags[i] = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         fence_proxy_async_smem();
     }
@@ -450,6 +457,30 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     break;
                 }
                 bool moved = false;
+                // Output products first: the softmax group of tile t2 waits for it before
+                // it can write its next P.
+                if (t2 < t1) {
+                    const int b = t2 & 1, s = t2 % kVStages;
+                    if (test_phase(&p_full[b], (t2 >> 1) & 1) && test_phase(&v_full[s], (t2 / kVStages) & 1)) {
+                        tc_fence_after();
+                        // O^T += V^T P into the group's accumulator; a group's first tile of
+                        // a segment starts it afresh.
+                        const uint32_t v0 = smem_u32(ringV + s * kTcHalfTile);
+                        const uint32_t p0 = smem_u32(sP + b * kTcPBytes);
+                        const uint32_t o = tmem + kTcOCol + b * kTcMaxCols;
+                        const uint32_t fresh = (t2 - starts[t2 % kSBufs]) < 2;
+#pragma unroll
+                        for (int k = 0; k < kTcRows / 16; ++k) {
+                            const uint64_t av = sdesc(v0 + k * 2048, kTcBox, 1024);
+                            umma(o, av, sdesc(p0 + k * 32, 16, 1024), id2, (fresh && k == 0) ? 0u : 1u);
+                            umma(o, av, sdesc(p0 + kTcMaxCols * 128 + k * 32, 16, 1024), id2, 1u);
+                        }
+                        umma_commit(smem_u32(&o_done[b]));
+                        umma_commit(smem_u32(&v_empty[s]));
+                        ++t2;
+                        moved = true;
+                    }
+                }
                 if (w1.more() && t1 < t2 + kSBufs) {
                     const int s = t1 % kKStages;
                     const bool first = w1.first();
@@ -475,28 +506,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         qseen = false;
                         ++t1;
                         w1.next(a, tab);
-                        moved = true;
-                    }
-                }
-                if (t2 < t1) {
-                    const int b = t2 & 1, s = t2 % kVStages;
-                    if (test_phase(&p_full[b], (t2 >> 1) & 1) && test_phase(&v_full[s], (t2 / kVStages) & 1)) {
-                        tc_fence_after();
-                        // O^T += V^T P into the group's accumulator; a group's first tile of
-                        // a segment starts it afresh.
-                        const uint32_t v0 = smem_u32(ringV + s * kTcHalfTile);
-                        const uint32_t p0 = smem_u32(sP + b * kTcPBytes);
-                        const uint32_t o = tmem + kTcOCol + b * kTcMaxCols;
-                        const uint32_t fresh = (t2 - starts[t2 % kSBufs]) < 2;
-#pragma unroll
-                        for (int k = 0; k < kTcRows / 16; ++k) {
-                            const uint64_t av = sdesc(v0 + k * 2048, kTcBox, 1024);
-                            umma(o, av, sdesc(p0 + k * 32, 16, 1024), id2, (fresh && k == 0) ? 0u : 1u);
-                            umma(o, av, sdesc(p0 + kTcMaxCols * 128 + k * 32, 16, 1024), id2, 1u);
-                        }
-                        umma_commit(smem_u32(&o_done[b]));
-                        umma_commit(smem_u32(&v_empty[s]));
-                        ++t2;
                         moved = true;
                     }
                 }
@@ -562,12 +571,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 const int cnt = w.cnt();
                 const bool gfirst = t - seg_start < 2;  // the group's first tile of the segment
                 last_mine = t;
-                // The tile's scores; the end of the group's previous output product (it
-                // read P buffer b, and rescaling O needs it done); for a partial tile,
-                // its V rows (zeroed below).
+                // The tile's scores (and, for a partial tile, its V rows, zeroed below).
+                // The end of the group's previous output product, which read P buffer b
+                // and wrote the group's O, is awaited once the scores are loaded (below),
+                // or here for the group's first tile of a segment, which has no vote.
                 if (gleader) {
                     bool ok = !flags[kFlagAbort] && wait_phase(&s_full[t % kSBufs], (t / kSBufs) & 1);
-                    if (ok && t >= 2) ok = wait_phase(&o_done[b], ((t - 2) >> 1) & 1);
+                    if (ok && gfirst && t >= 2) ok = wait_phase(&o_done[b], ((t - 2) >> 1) & 1);
                     if (ok && cnt < kTcRows) ok = wait_phase(&v_full[t % kVStages], (t / kVStages) & 1);
                     if (!ok && !flags[kFlagAbort]) {
                         atomicOr(a.status, kDevTmaTimeout);
@@ -595,18 +605,30 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                                      fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
                     mt = fmaxf(mt, __shfl_xor_sync(kFull, mt, 16));  // the column's other half
                     mt = live ? mt * cs : -INFINITY;  // scale > 0: the max of the scaled scores
+                    bool go = true;
                     if (gfirst) {
                         m = mt;
                         l = 0.f;
                     } else {
-                        // Lazy rescale: only when a column's tile max tops its running max by kSlack.
-                        const bool vote = live && mt > m + kSlack;
+                        // Lazy rescale: only when a column's tile max tops its running max by kSlackTc.
+                        const bool vote = live && mt > m + kSlackTc;
                         const unsigned any = __ballot_sync(kFull, vote);
                         if (lane == 0) flags[kFlagVote + 4 * gi + quarter] = any != 0;
+                        if (gleader) {
+                            bool ok = t < 2 || wait_phase(&o_done[b], ((t - 2) >> 1) & 1);
+                            if (!ok && !flags[kFlagAbort]) {
+                                atomicOr(a.status, kDevTmaTimeout);
+                                flags[kFlagAbort] = 1;
+                            }
+                            flags[kFlagOk2 + gi] = ok;
+                            tc_fence_before();
+                        }
                         named_sync(gbar, kTcGroup);
+                        go = flags[kFlagOk2 + gi];
+                        tc_fence_after();
                         const bool rescale = flags[kFlagVote + 4 * gi] | flags[kFlagVote + 4 * gi + 1] |
                                              flags[kFlagVote + 4 * gi + 2] | flags[kFlagVote + 4 * gi + 3];
-                        if (rescale) {
+                        if (go && rescale) {
                             float alpha = 1.f;
                             if (vote) {
                                 alpha = ex2(m - mt);
@@ -626,46 +648,48 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                             }
                         }
                     }
-                    // P = 2^(s - m): a bf16 high part (the top 16 bits) and the bf16 of
-                    // the remainder, row col of the B operand (64 rows, 128 bytes, swizzled).
-                    if (col < NCpad) {
-                        // Columns past NC get p = 0: 2^(s - inf) = 0 for finite or -inf s.
-                        const float nm = live ? -m : -INFINITY;
-                        unsigned char* ph = sP + b * kTcPBytes + col * 128;
-                        unsigned char* pl = ph + kTcMaxCols * 128;
-                        float ls[4] = {0.f, 0.f, 0.f, 0.f};
+                    if (go) {
+                        // P = 2^(s - m): a bf16 high part (the top 16 bits) and the bf16 of
+                        // the remainder, row col of the B operand (64 rows, 128 bytes, swizzled).
+                        if (col < NCpad) {
+                            // Columns past NC get p = 0: 2^(s - inf) = 0 for finite or -inf s.
+                            const float nm = live ? -m : -INFINITY;
+                            unsigned char* ph = sP + b * kTcPBytes + col * 128;
+                            unsigned char* pl = ph + kTcMaxCols * 128;
+                            float ls[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-                        for (int ch = 0; ch < 4; ++ch) {
-                            uint32_t hi[4], lo[4];
+                            for (int ch = 0; ch < 4; ++ch) {
+                                uint32_t hi[4], lo[4];
 #pragma unroll
-                            for (int i = 0; i < 4; ++i) {
-                                const float p0 = ex2(fmaf(sc[8 * ch + 2 * i], cs, nm));  // 2^-inf = 0
-                                const float p1 = ex2(fmaf(sc[8 * ch + 2 * i + 1], cs, nm));
-                                ls[i] += p0 + p1;
-                                const uint32_t h0 = __float_as_uint(p0) & 0xffff0000u;
-                                const uint32_t h1 = __float_as_uint(p1) & 0xffff0000u;
-                                hi[i] = __byte_perm(h0, h1, 0x7632);
-                                lo[i] = pack_bf16(p0 - __uint_as_float(h0), p1 - __uint_as_float(h1));
+                                for (int i = 0; i < 4; ++i) {
+                                    const float p0 = ex2(fmaf(sc[8 * ch + 2 * i], cs, nm));  // 2^-inf = 0
+                                    const float p1 = ex2(fmaf(sc[8 * ch + 2 * i + 1], cs, nm));
+                                    ls[i] += p0 + p1;
+                                    const uint32_t h0 = __float_as_uint(p0) & 0xffff0000u;
+                                    const uint32_t h1 = __float_as_uint(p1) & 0xffff0000u;
+                                    hi[i] = __byte_perm(h0, h1, 0x7632);
+                                    lo[i] = pack_bf16(p0 - __uint_as_float(h0), p1 - __uint_as_float(h1));
+                                }
+                                const int off = ((4 * half + ch) ^ (col & 7)) << 4;
+                                *reinterpret_cast<uint4*>(ph + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+                                *reinterpret_cast<uint4*>(pl + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
                             }
-                            const int off = ((4 * half + ch) ^ (col & 7)) << 4;
-                            *reinterpret_cast<uint4*>(ph + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-                            *reinterpret_cast<uint4*>(pl + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+                            l += (ls[0] + ls[1]) + (ls[2] + ls[3]);
                         }
-                        l += (ls[0] + ls[1]) + (ls[2] + ls[3]);
-                    }
-                    if (cnt < kTcRows) {
-                        // V rows past the segment: zeros (their p is 0, but 0 * inf or 0 * nan would not be).
-                        unsigned char* v0 = ringV + (t % kVStages) * kTcHalfTile;
-                        for (int i = gt; i < (kTcRows - cnt) * 16; i += kTcGroup) {
-                            const int r = cnt + (i >> 4), k = i & 15;
-                            *reinterpret_cast<uint4*>(v0 + (k >> 3) * kTcBox + r * 128 + ((k & 7) << 4)) =
-                                make_uint4(0u, 0u, 0u, 0u);
+                        if (cnt < kTcRows) {
+                            // V rows past the segment: zeros (their p is 0, but 0 * inf or 0 * nan would not be).
+                            unsigned char* v0 = ringV + (t % kVStages) * kTcHalfTile;
+                            for (int i = gt; i < (kTcRows - cnt) * 16; i += kTcGroup) {
+                                const int r = cnt + (i >> 4), k = i & 15;
+                                *reinterpret_cast<uint4*>(v0 + (k >> 3) * kTcBox + r * 128 + ((k & 7) << 4)) =
+                                    make_uint4(0u, 0u, 0u, 0u);
+                            }
                         }
+                        fence_proxy_async_smem();
+                        tc_fence_before();
+                        named_sync(gbar, kTcGroup);
+                        if (gleader) mbar_arrive(smem_u32(&p_full[b]));
                     }
-                    fence_proxy_async_smem();
-                    tc_fence_before();
-                    named_sync(gbar, kTcGroup);
-                    if (gleader) mbar_arrive(smem_u32(&p_full[b]));
                 }
             }
             if (!last) continue;
@@ -732,11 +756,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     }
                 }
             }
-            if (merge_ok && !whole) __threadfence();  // the partial, before the count below
             // g_max / g_sum are rewritten at the next segment's end, after these reads.
             named_sync(kBarSoft, kTcSoft);
             if (merge_ok && !whole && leader) {
-                // This CTA's partial of slab h is written: count it in.
+                // This CTA's partial of slab h is written (the barrier above orders the
+                // other threads' stores before this thread's fence): count it in.
                 __threadfence();
                 atomicAdd(a.slab_count + (int64_t)h * kMaxCols * 2, 1);
             }
