@@ -20,8 +20,9 @@
 //                       to four tiles ahead of O^T += V^T P  (M = 128 dims, N =
 //                       the columns rounded up to 16, K = 64 rows; V^T read
 //                       MN-major from its stage; P as a bf16 high part and
-//                       remainder, two MMAs per k-step) into the TMEM output
-//                       accumulator of the tile's softmax group.
+//                       remainder side by side, N = 2 x the columns, one MMA per
+//                       k-step) into the TMEM output accumulator of the tile's
+//                       softmax group, whose two halves are summed when read.
 //   warps 2-5, 6-9      two softmax groups; group g takes the tiles t with
 //                       t % 2 == g, with its own running max and sum of every
 //                       column and its own O accumulator (merged at a segment's
@@ -72,9 +73,10 @@ constexpr int kTcGroup = 128;                  // threads of one softmax group
 constexpr int kTcQRows = 64;                   // M of the score product: the most columns
 constexpr int kTcQHalf = kTcQRows * 128;       // one 64-dim half of Q (8 KB)
 constexpr int kTcQBytes = 2 * kTcQHalf;        // Q as the A operand: 64 rows x 128 dims (two buffers: segments alternate)
-constexpr int kTcPBytes = 2 * kTcMaxCols * 128;  // one P buffer: high and low parts, 64 columns x 64 rows each
+constexpr int kTcPBytes = 2 * kTcMaxCols * 128;  // one P buffer: high parts (rows 0..NCpad-1), then low parts, 64 rows each
 constexpr int kSBufs = 4;                      // TMEM score buffers
-constexpr int kTcTmemCols = 512;               // S buffers at columns 0, 64, 128, 192; O of group g at 256 + 64 g
+constexpr int kTcTmemCols = 512;               // S buffers at columns 0, 64, 128, 192; O of group g at 256 + 128 g
+constexpr int kTcOCols = 2 * kTcMaxCols;       // O of one group: the product with P's high parts, then with its low parts
 constexpr int kTcOCol = kSBufs * kTcRows;
 // Named barriers: 1 + g for softmax group g, kBarSoft for both groups, kBarTmem for warps 1-9.
 constexpr int kBarSoft = 3, kBarTmem = 4;
@@ -442,7 +444,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         // the segment's Q; an output product needs its P and its V stage.
         if (lane == 0) {
             const uint32_t id1 = idesc(kTcQRows, kTcRows, 0, 0);
-            const uint32_t id2 = idesc(128, NCpad, 1, 0);
+            const uint32_t id2 = idesc(128, 2 * NCpad, 1, 0);  // high and low parts of P side by side
             TileWalk w1;
             w1.begin(a, tab, hfirst, hend, A, Bc);
             int t1 = 0, t2 = 0, seg = 0, seg_start = 0;
@@ -463,18 +465,17 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     const int b = t2 & 1, s = t2 % kVStages;
                     if (test_phase(&p_full[b], (t2 >> 1) & 1) && test_phase(&v_full[s], (t2 / kVStages) & 1)) {
                         tc_fence_after();
-                        // O^T += V^T P into the group's accumulator; a group's first tile of
-                        // a segment starts it afresh.
+                        // O^T += V^T [P_hi P_lo] into the group's accumulator (the two
+                        // halves are summed when O is read); a group's first tile of a
+                        // segment starts it afresh.
                         const uint32_t v0 = smem_u32(ringV + s * kTcHalfTile);
                         const uint32_t p0 = smem_u32(sP + b * kTcPBytes);
-                        const uint32_t o = tmem + kTcOCol + b * kTcMaxCols;
+                        const uint32_t o = tmem + kTcOCol + b * kTcOCols;
                         const uint32_t fresh = (t2 - starts[t2 % kSBufs]) < 2;
 #pragma unroll
-                        for (int k = 0; k < kTcRows / 16; ++k) {
-                            const uint64_t av = sdesc(v0 + k * 2048, kTcBox, 1024);
-                            umma(o, av, sdesc(p0 + k * 32, 16, 1024), id2, (fresh && k == 0) ? 0u : 1u);
-                            umma(o, av, sdesc(p0 + kTcMaxCols * 128 + k * 32, 16, 1024), id2, 1u);
-                        }
+                        for (int k = 0; k < kTcRows / 16; ++k)
+                            umma(o, sdesc(v0 + k * 2048, kTcBox, 1024), sdesc(p0 + k * 32, 16, 1024), id2,
+                                 (fresh && k == 0) ? 0u : 1u);
                         umma_commit(smem_u32(&o_done[b]));
                         umma_commit(smem_u32(&v_empty[s]));
                         ++t2;
@@ -536,7 +537,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const int col = 16 * quarter + (lane & 15);
         const bool live = col < NC;
         const int dim = 32 * quarter + lane;
-        const uint32_t my_o = tmem + lane_addr + kTcOCol + gi * kTcMaxCols;
+        const uint32_t my_o = tmem + lane_addr + kTcOCol + gi * kTcOCols;
         pdl_wait();  // q and the outputs belong to the previous kernel's epoch
         TileWalk w;
         w.begin(a, tab, hfirst, hend, A, Bc);
@@ -637,13 +638,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                             }
                             if (half == 0) g_alpha[gi * kTcMaxCols + col] = alpha;
                             named_sync(gbar, kTcGroup);
-                            // The group's O (its previous product is done: waited above).
-                            for (int c0 = 0; c0 < NCpad; c0 += 32) {
+                            // The group's O, both halves (its previous product is done: waited above).
+                            for (int c0 = 0; c0 < 2 * NCpad; c0 += 32) {
                                 float v[32];
                                 tmem_ld32(my_o + c0, v);
 #pragma unroll
-                                for (int i = 0; i < 32; ++i)
-                                    v[i] *= (c0 + i < NC) ? g_alpha[gi * kTcMaxCols + c0 + i] : 1.f;
+                                for (int i = 0; i < 32; ++i) {
+                                    const int cc = c0 + i < NCpad ? c0 + i : c0 + i - NCpad;
+                                    v[i] *= cc < NC ? g_alpha[gi * kTcMaxCols + cc] : 1.f;
+                                }
                                 tmem_st32(my_o + c0, v);
                             }
                         }
@@ -655,7 +658,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                             // Columns past NC get p = 0: 2^(s - inf) = 0 for finite or -inf s.
                             const float nm = live ? -m : -INFINITY;
                             unsigned char* ph = sP + b * kTcPBytes + col * 128;
-                            unsigned char* pl = ph + kTcMaxCols * 128;
+                            unsigned char* pl = ph + NCpad * 128;  // row NCpad + col: same swizzle phase
                             float ls[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
                             for (int ch = 0; ch < 4; ++ch) {
@@ -736,9 +739,20 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             const int bq = h / a.Hkv, g = h - bq * a.Hkv;
             const int64_t slot = (int64_t)c + h;
             if (merge_ok && oc0 < NCpad) {
+                // O of each group = its product with P_hi + its product with P_lo.
                 float v0[32], v1[32];
-                tmem_ld32(tmem + lane_addr + kTcOCol + oc0, v0);
-                tmem_ld32(tmem + lane_addr + kTcOCol + kTcMaxCols + oc0, v1);
+                {
+                    float w[32];
+                    const uint32_t o0 = tmem + lane_addr + kTcOCol, o1 = o0 + kTcOCols;
+                    tmem_ld32(o0 + oc0, v0);
+                    tmem_ld32(o0 + NCpad + oc0, w);
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) v0[i] += w[i];
+                    tmem_ld32(o1 + oc0, v1);
+                    tmem_ld32(o1 + NCpad + oc0, w);
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) v1[i] += w[i];
+                }
 #pragma unroll
                 for (int i = 0; i < 32; ++i) {
                     const int cc = oc0 + i;
