@@ -44,9 +44,11 @@ from paper_2609_32663_gb300 import inputs as I  # noqa: E402
 DECODE_TRAFFIC = {
     "sources": ("paper_2609_32663_gb300/csrc/dkv_decode_mma.cu", "paper_2609_32663_gb300/csrc/dkv_decode_common.cuh",
                 "paper_2609_32663_gb300/csrc/dkv_ptx.cuh", "paper_2609_32663_gb300/csrc/dkv_internal.cuh"),
-    "sha256": None,  # the kernel changed since the capture: traffic unknown until re-captured
-    "dram_bytes": 194_384_896 + 3_126_272,
-    "algorithmic_bytes": 376_646 * 512 + 32 * 128 * (2 + 4),
+    "sha256": "e5d64f39513c799e4719fa1a394bcae43514f0d073a6c583b639c60beb37cbfe",
+    # ncu of decode_mma_kernel<4, 1, 1, 0>, llama8b-128k-l4, the 13th launch (layer 0
+    # with 2 rows appended before it and one by it: 376,646 + 8 x 3 rows)
+    "dram_bytes": 194_374_656 + 3_159_040,
+    "algorithmic_bytes": 376_670 * 512 + 32 * (256 + 512) + 4 * 8 * 256,
 }
 
 

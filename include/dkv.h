@@ -264,11 +264,20 @@ dkv_status dkv_decode_attn(const dkv_plan* plan, int32_t layer, const void* q,
  *
  * q    device bf16 [B][num_queries][H][128].
  * out  device fp32 [B][num_queries][H][128].
- * Needs 1 <= num_queries and num_queries * G <= 16 (G = H / H_kv), and a plan
+ * Needs 1 <= num_queries and num_queries * G <= 64 (G = H / H_kv), and a plan
  * whose cache has fewer than 2^31 rows. The query x head columns of a KV head
- * are the n side of one tensor-core product per tile of 16 rows, so the K/V
- * rows are read once for all queries. Other arguments, ordering and errors are
- * those of dkv_decode_attn.
+ * (num_queries * G of them) share every K/V row, so the rows are read once for
+ * all queries:
+ *   <= 16 columns  a split-K kernel whose warps multiply 16-row tiles on the
+ *                  warp-level tensor-core path, then a combine kernel;
+ *   17..64         one tcgen05 kernel: 64-row tiles staged by TMA, scores and
+ *                  outputs accumulated in tensor memory, and the CTAs that
+ *                  share a slab merge their partials inside the same launch.
+ *                  It is a cooperative launch (all CTAs resident at once), so
+ *                  it fails with DKV_ERR_CUDA where the device cannot grant
+ *                  one (for example under a partitioned device).
+ * Other arguments, ordering and errors are those of dkv_decode_attn; a
+ * num_queries * G above 64 is DKV_ERR_INVALID_ARG.
  */
 dkv_status dkv_decode_multi(const dkv_plan* plan, int32_t layer, const void* q, int32_t num_queries,
                             const int32_t* n_appended, void* Kc, void* Vc, float scale, float* out,
