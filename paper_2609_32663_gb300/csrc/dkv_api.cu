@@ -675,7 +675,7 @@ dkv_status dkv_decode_multi(const dkv_plan* p, int32_t layer, const void* q, int
         // tcgen05 kernel (accumulators in TMEM).
         a.nctas = p->cfg_tc.nctas;
         dkv::CacheMaps maps;
-        const cudaError_t e = dkv::make_cache_maps(a.Kc, a.Vc, p->total_rows, &maps, fault("copy"), 64);
+        const cudaError_t e = dkv::make_cache_maps(a.Kc, a.Vc, p->total_rows, &maps, fault("copy"), 16);
         if (e != cudaSuccess) return cuda_fail(e, "tensor maps of the packed caches");
         st = launched(dkv::launch_decode_tc(a, maps, p->cfg_tc, stream), "multi-query decode kernel (tcgen05)");
         return st == DKV_OK ? ok() : st;

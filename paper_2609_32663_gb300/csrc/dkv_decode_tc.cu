@@ -9,8 +9,9 @@
 // kernels; a CTA walks its range in tiles of 64 rows, slab segment by slab
 // segment (a segment: the part of one slab inside the CTA's range).
 //
-//   warp 0 (one lane)   TMA: a tile's K rows and V rows, each as two 2-D boxes
-//                       (64 rows x 64 dims, 128-byte swizzle), into separate
+//   warp 0 (one lane)   TMA: a tile's K rows and V rows, each as 16-row 2-D
+//                       boxes (64 dims, 128-byte swizzle; measured faster than
+//                       64- or 32-row boxes), into separate
 //                       rings (4 K stages, 5 V stages): a K stage is released as
 //                       soon as its score product is done, a V stage only after
 //                       its output product, so V is the deeper ring.
@@ -65,7 +66,8 @@ namespace {
 constexpr int kTcRows = 64;                    // cache rows per tile
 constexpr int kKStages = 4;                    // K ring stages
 constexpr int kVStages = 5;                    // V ring stages
-constexpr int kTcBox = kTcRows * 128;          // one TMA box: 64 rows x 64 dims of bf16 (8 KB)
+constexpr int kTcBox = kTcRows * 128;          // one 64-dim half of a tile: 64 rows x 64 dims of bf16 (8 KB)
+constexpr int kTcBoxRows = 16;                 // rows of one TMA box (measured: 16-row boxes beat 64- and 32-row ones)
 constexpr int kTcHalfTile = 2 * kTcBox;        // K (or V) rows of one tile: dims 0-63, then 64-127
 constexpr int kTcThreads = 320;                // warps: 0 TMA, 1 MMA, 2-5 and 6-9 the two softmax groups
 constexpr int kTcSoft = 256;                   // threads of the softmax warps
@@ -395,8 +397,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     const int s = tk % kKStages, row = wk.cache_row();
                     const uint32_t bar = smem_u32(&k_full[s]), dst = smem_u32(ringK + s * kTcHalfTile);
                     mbar_arrive_expect_tx(bar, kTcHalfTile);
-                    tma_box(dst, &maps.k, 0, row, bar, pol);
-                    tma_box(dst + kTcBox, &maps.k, 64, row, bar, pol);
+#pragma unroll
+                    for (int j = 0; j < kTcRows / kTcBoxRows; ++j) {
+                        tma_box(dst + j * kTcBoxRows * 128, &maps.k, 0, row + j * kTcBoxRows, bar, pol);
+                        tma_box(dst + kTcBox + j * kTcBoxRows * 128, &maps.k, 64, row + j * kTcBoxRows, bar, pol);
+                    }
                     ++tk;
                     wk.next(a, tab);
                     moved = true;
@@ -405,8 +410,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     const int s = tv % kVStages, row = wv.cache_row();
                     const uint32_t bar = smem_u32(&v_full[s]), dst = smem_u32(ringV + s * kTcHalfTile);
                     mbar_arrive_expect_tx(bar, kTcHalfTile);
-                    tma_box(dst, &maps.v, 0, row, bar, pol);
-                    tma_box(dst + kTcBox, &maps.v, 64, row, bar, pol);
+#pragma unroll
+                    for (int j = 0; j < kTcRows / kTcBoxRows; ++j) {
+                        tma_box(dst + j * kTcBoxRows * 128, &maps.v, 0, row + j * kTcBoxRows, bar, pol);
+                        tma_box(dst + kTcBox + j * kTcBoxRows * 128, &maps.v, 64, row + j * kTcBoxRows, bar, pol);
+                    }
                     ++tv;
                     wv.next(a, tab);
                     moved = true;
@@ -445,19 +453,25 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         if (lane == 0) {
             const uint32_t id1 = idesc(kTcQRows, kTcRows, 0, 0);
             const uint32_t id2 = idesc(128, 2 * NCpad, 1, 0);  // high and low parts of P side by side
+            // Operand descriptors of the first stage of each ring; a stage or k-step
+            // further on is a constant added to the address field (16-byte units; every
+            // shared-memory address is below 2^18 bytes, so the 14-bit field never
+            // carries). One thread issues every product, so its per-product work is the
+            // pipeline's pace: nothing is recomputed per k-step.
+            const uint64_t dQ = sdesc(smem_u32(sQ), 16, 1024);
+            const uint64_t dK = sdesc(smem_u32(ringK), 16, 1024);
+            const uint64_t dV = sdesc(smem_u32(ringV), kTcBox, 1024);
+            const uint64_t dP = sdesc(smem_u32(sP), 16, 1024);
             TileWalk w1;
             w1.begin(a, tab, hfirst, hend, A, Bc);
             int t1 = 0, t2 = 0, seg = 0, seg_start = 0;
-            // Segment start of tiles between the two products (at most kSBufs).
-            int starts[kSBufs] = {0, 0, 0, 0};
+            // Bit t % kSBufs: tile t (between the two products) is one of the first two
+            // of its segment, so its group's output product starts the accumulator afresh.
+            uint32_t fresh_bits = 0;
             int qbuf = 0;  // Q buffer of the segment of tile t1
             bool issued = false, ok = true, qseen = false;
             IdleBound idle;
-            while ((w1.more() || t2 < t1) && ok) {
-                if (flags[kFlagAbort]) {
-                    ok = false;
-                    break;
-                }
+            while (w1.more() || t2 < t1) {
                 bool moved = false;
                 // Output products first: the softmax group of tile t2 waits for it before
                 // it can write its next P.
@@ -468,14 +482,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         // O^T += V^T [P_hi P_lo] into the group's accumulator (the two
                         // halves are summed when O is read); a group's first tile of a
                         // segment starts it afresh.
-                        const uint32_t v0 = smem_u32(ringV + s * kTcHalfTile);
-                        const uint32_t p0 = smem_u32(sP + b * kTcPBytes);
+                        const uint64_t va = dV + (uint64_t)(s * (kTcHalfTile >> 4));
+                        const uint64_t pb = dP + (uint64_t)(b * (kTcPBytes >> 4));
                         const uint32_t o = tmem + kTcOCol + b * kTcOCols;
-                        const uint32_t fresh = (t2 - starts[t2 % kSBufs]) < 2;
+                        const uint32_t fresh = (fresh_bits >> (t2 % kSBufs)) & 1u;
+                        umma(o, va, pb, id2, fresh ^ 1u);
 #pragma unroll
-                        for (int k = 0; k < kTcRows / 16; ++k)
-                            umma(o, sdesc(v0 + k * 2048, kTcBox, 1024), sdesc(p0 + k * 32, 16, 1024), id2,
-                                 (fresh && k == 0) ? 0u : 1u);
+                        for (int k = 1; k < kTcRows / 16; ++k)
+                            umma(o, va + (uint64_t)(k * (2048 >> 4)), pb + (uint64_t)(k * (32 >> 4)), id2, 1u);
                         umma_commit(smem_u32(&o_done[b]));
                         umma_commit(smem_u32(&v_empty[s]));
                         ++t2;
@@ -493,16 +507,19 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     }
                     if ((!first || qseen) && test_phase(&k_full[s], (t1 / kKStages) & 1)) {
                         tc_fence_after();
-                        // S^T[64 x 64] = Q[64 x 128] K^T: k-steps of 16 dims (+32 B inside a 64-dim half).
-                        const uint32_t q0 = smem_u32(sQ + qbuf * kTcQBytes), k0 = smem_u32(ringK + s * kTcHalfTile);
+                        // S^T[64 x 64] = Q[64 x 128] K^T: k-steps of 16 dims (+32 B inside a
+                        // 64-dim half, +kTcBox or +kTcQHalf to the next half).
+                        const uint64_t qa = dQ + (uint64_t)(qbuf * (kTcQBytes >> 4));
+                        const uint64_t kb = dK + (uint64_t)(s * (kTcHalfTile >> 4));
                         const uint32_t d = tmem + (t1 % kSBufs) * kTcRows;
 #pragma unroll
                         for (int k = 0; k < 8; ++k)
-                            umma(d, sdesc(q0 + (k >> 2) * kTcQHalf + (k & 3) * 32, 16, 1024),
-                                 sdesc(k0 + (k >> 2) * kTcBox + (k & 3) * 32, 16, 1024), id1, k > 0 ? 1u : 0u);
+                            umma(d, qa + (uint64_t)((k >> 2) * (kTcQHalf >> 4) + (k & 3) * 2),
+                                 kb + (uint64_t)((k >> 2) * (kTcBox >> 4) + (k & 3) * 2), id1, k > 0 ? 1u : 0u);
                         umma_commit(smem_u32(&s_full[t1 % kSBufs]));
                         umma_commit(smem_u32(&k_empty[s]));
-                        starts[t1 % kSBufs] = seg_start;
+                        const uint32_t bit = 1u << (t1 % kSBufs);
+                        fresh_bits = (t1 - seg_start < 2) ? (fresh_bits | bit) : (fresh_bits & ~bit);
                         issued = true;
                         qseen = false;
                         ++t1;
@@ -512,8 +529,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 }
                 if (moved) {
                     idle.progress();
-                } else if (idle.expired()) {
+                } else if (flags[kFlagAbort] || idle.expired()) {
+                    // Another role gave up, or nothing moved within the bound.
                     ok = false;
+                    break;
                 } else {
                     __nanosleep(20);
                 }
