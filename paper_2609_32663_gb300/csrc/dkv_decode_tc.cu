@@ -189,6 +189,36 @@ __device__ __forceinline__ void tmem_ld16x2(uint32_t taddr, float (&v)[32])
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// 16 consecutive TMEM columns of this thread's lane, without the wait: the
+// registers are valid only after tmem_wait_ld, which takes them as operands so
+// that no use of them can be scheduled before it.
+__device__ __forceinline__ void tmem_ld16_async(uint32_t taddr, uint32_t (&r)[16])
+{
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+}
+
+__device__ __forceinline__ void tmem_fence_regs(uint32_t (&r)[16])
+{
+    asm volatile(""
+                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
+                   "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]),
+                   "+r"(r[15]));
+}
+
+__device__ __forceinline__ void tmem_wait_ld(uint32_t (&a)[16], uint32_t (&b)[16], uint32_t (&c)[16],
+                                             uint32_t (&d)[16])
+{
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+    tmem_fence_regs(a);
+    tmem_fence_regs(b);
+    tmem_fence_regs(c);
+    tmem_fence_regs(d);
+}
+
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const float (&v)[32])
 {
     asm volatile(
@@ -758,34 +788,36 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             const int bq = h / a.Hkv, g = h - bq * a.Hkv;
             const int64_t slot = (int64_t)c + h;
             if (merge_ok && oc0 < NCpad) {
-                // O of each group = its product with P_hi + its product with P_lo.
-                float v0[32], v1[32];
-                {
-                    float w[32];
-                    const uint32_t o0 = tmem + lane_addr + kTcOCol, o1 = o0 + kTcOCols;
-                    tmem_ld32(o0 + oc0, v0);
-                    tmem_ld32(o0 + NCpad + oc0, w);
+                // O of each group = its product with P_hi + its product with P_lo, 16
+                // columns at a time (whole 32-column blocks spilled registers to local
+                // memory, which misses the small L1 left beside this kernel's shared
+                // memory and cost microseconds per segment end).
+                const uint32_t o0 = tmem + lane_addr + kTcOCol, o1 = o0 + kTcOCols;
+#pragma unroll 1
+                for (int c16 = oc0; c16 < oc0 + 32 && c16 < NC; c16 += 16) {
+                    uint32_t r0[16], w0[16], r1[16], w1[16];
+                    tmem_ld16_async(o0 + c16, r0);
+                    tmem_ld16_async(o0 + NCpad + c16, w0);
+                    tmem_ld16_async(o1 + c16, r1);
+                    tmem_ld16_async(o1 + NCpad + c16, w1);
+                    tmem_wait_ld(r0, w0, r1, w1);
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) v0[i] += w[i];
-                    tmem_ld32(o1 + oc0, v1);
-                    tmem_ld32(o1 + NCpad + oc0, w);
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) v1[i] += w[i];
-                }
-#pragma unroll
-                for (int i = 0; i < 32; ++i) {
-                    const int cc = oc0 + i;
-                    if (cc >= NC) break;
-                    const float m0 = has0 ? g_max[cc] : -INFINITY, m1 = has1 ? g_max[kTcMaxCols + cc] : -INFINITY;
-                    const float M = fmaxf(m0, m1);
-                    const float f0 = has0 ? ex2(m0 - M) : 0.f, f1 = has1 ? ex2(m1 - M) : 0.f;
-                    const float o = (has0 ? f0 * v0[i] : 0.f) + (has1 ? f1 * v1[i] : 0.f);
-                    const float L = (has0 ? f0 * g_sum[cc] : 0.f) + (has1 ? f1 * g_sum[kTcMaxCols + cc] : 0.f);
-                    if (whole) {
-                        a.out[out_row<G>(a, bq, g, cc) * kHeadDim + dim] = L > 0.f ? o / L : 0.f;
-                    } else {
-                        a.work_o[(slot * NC + cc) * kHeadDim + dim] = o;
-                        if (dim == 0) *reinterpret_cast<float2*>(a.work_ml + (slot * NC + cc) * 2) = make_float2(M, L);
+                    for (int i = 0; i < 16; ++i) {
+                        const int cc = c16 + i;
+                        if (cc >= NC) break;
+                        const float m0 = has0 ? g_max[cc] : -INFINITY, m1 = has1 ? g_max[kTcMaxCols + cc] : -INFINITY;
+                        const float M = fmaxf(m0, m1);
+                        const float f0 = has0 ? ex2(m0 - M) : 0.f, f1 = has1 ? ex2(m1 - M) : 0.f;
+                        const float v0 = __uint_as_float(r0[i]) + __uint_as_float(w0[i]);
+                        const float v1 = __uint_as_float(r1[i]) + __uint_as_float(w1[i]);
+                        const float o = (has0 ? f0 * v0 : 0.f) + (has1 ? f1 * v1 : 0.f);
+                        const float L = (has0 ? f0 * g_sum[cc] : 0.f) + (has1 ? f1 * g_sum[kTcMaxCols + cc] : 0.f);
+                        if (whole) {
+                            a.out[out_row<G>(a, bq, g, cc) * kHeadDim + dim] = L > 0.f ? o / L : 0.f;
+                        } else {
+                            a.work_o[(slot * NC + cc) * kHeadDim + dim] = o;
+                            if (dim == 0) *reinterpret_cast<float2*>(a.work_ml + (slot * NC + cc) * 2) = make_float2(M, L);
+                        }
                     }
                 }
             }
