@@ -801,22 +801,34 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     tmem_ld16_async(o1 + c16, r1);
                     tmem_ld16_async(o1 + NCpad + c16, w1);
                     tmem_wait_ld(r0, w0, r1, w1);
+                    // Columns up to c16 + 15 are read even past NC (the statistics arrays
+                    // hold kTcMaxCols columns), so that every shared-memory load of the
+                    // chunk is independent of the stores: a load-use chain per column
+                    // cost ~250 cycles a column under the kernel's shared-memory traffic.
+                    float ov[16], Mv[16], Lv[16];
 #pragma unroll
                     for (int i = 0; i < 16; ++i) {
                         const int cc = c16 + i;
-                        if (cc >= NC) break;
                         const float m0 = has0 ? g_max[cc] : -INFINITY, m1 = has1 ? g_max[kTcMaxCols + cc] : -INFINITY;
                         const float M = fmaxf(m0, m1);
                         const float f0 = has0 ? ex2(m0 - M) : 0.f, f1 = has1 ? ex2(m1 - M) : 0.f;
                         const float v0 = __uint_as_float(r0[i]) + __uint_as_float(w0[i]);
                         const float v1 = __uint_as_float(r1[i]) + __uint_as_float(w1[i]);
-                        const float o = (has0 ? f0 * v0 : 0.f) + (has1 ? f1 * v1 : 0.f);
-                        const float L = (has0 ? f0 * g_sum[cc] : 0.f) + (has1 ? f1 * g_sum[kTcMaxCols + cc] : 0.f);
-                        if (whole) {
-                            a.out[out_row<G>(a, bq, g, cc) * kHeadDim + dim] = L > 0.f ? o / L : 0.f;
-                        } else {
-                            a.work_o[(slot * NC + cc) * kHeadDim + dim] = o;
-                            if (dim == 0) *reinterpret_cast<float2*>(a.work_ml + (slot * NC + cc) * 2) = make_float2(M, L);
+                        ov[i] = (has0 ? f0 * v0 : 0.f) + (has1 ? f1 * v1 : 0.f);
+                        Mv[i] = M;
+                        Lv[i] = (has0 ? f0 * g_sum[cc] : 0.f) + (has1 ? f1 * g_sum[kTcMaxCols + cc] : 0.f);
+                    }
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        const int cc = c16 + i;
+                        if (cc < NC) {
+                            if (whole) {
+                                a.out[out_row<G>(a, bq, g, cc) * kHeadDim + dim] = Lv[i] > 0.f ? ov[i] / Lv[i] : 0.f;
+                            } else {
+                                a.work_o[(slot * NC + cc) * kHeadDim + dim] = ov[i];
+                                if (dim == 0)
+                                    *reinterpret_cast<float2*>(a.work_ml + (slot * NC + cc) * 2) = make_float2(Mv[i], Lv[i]);
+                            }
                         }
                     }
                 }
