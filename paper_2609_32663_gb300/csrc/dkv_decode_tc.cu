@@ -463,6 +463,23 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             flags[kFlagVIssued] = tv;
         }
     } else {
+        if (warp >= 2) {
+            // The first two segments' Q (buffers 0 and 1), loaded while warp 1
+            // allocates TMEM: the first score product waits for both.
+            const int st = tid - 64;
+            pdl_wait();  // q and the outputs belong to the previous kernel's epoch
+            TileWalk w0;
+            w0.begin(a, tab, hfirst, hend, A, Bc);
+            const int h1 = later_segment_slab(w0.cu, a, tab, hend, A, Bc, 1);
+            load_q_tc<G>(a, w0.cu.h, sQ, st);
+            if (h1 < hend) load_q_tc<G>(a, h1, sQ + kTcQBytes, st);
+            fence_proxy_async_smem();
+            named_sync(kBarSoft, kTcSoft);
+            if (st == 0) {
+                mbar_arrive(smem_u32(&q_full[0]));
+                if (h1 < hend) mbar_arrive(smem_u32(&q_full[1]));
+            }
+        }
         if (warp == 1) {
             asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
                          "r"(kTcTmemCols));
@@ -587,19 +604,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const bool live = col < NC;
         const int dim = 32 * quarter + lane;
         const uint32_t my_o = tmem + lane_addr + kTcOCol + gi * kTcOCols;
-        pdl_wait();  // q and the outputs belong to the previous kernel's epoch
         TileWalk w;
         w.begin(a, tab, hfirst, hend, A, Bc);
-        // Q of the first two segments (buffers 0 and 1).
-        const int h1 = later_segment_slab(w.cu, a, tab, hend, A, Bc, 1);
-        load_q_tc<G>(a, w.cu.h, sQ, st);
-        if (h1 < hend) load_q_tc<G>(a, h1, sQ + kTcQBytes, st);
-        fence_proxy_async_smem();
-        named_sync(kBarSoft, kTcSoft);
-        if (leader) {
-            mbar_arrive(smem_u32(&q_full[0]));
-            if (h1 < hend) mbar_arrive(smem_u32(&q_full[1]));
-        }
         int seg_idx = -1;              // index of the current segment
         float m = -INFINITY, l = 0.f;  // this group's running max (log2 units) and sum of column col
         int t = 0, seg_start = 0;
@@ -888,34 +894,37 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 const int j0 = (int)((int64_t)k * NC / nct), j1 = (int)((int64_t)(k + 1) * NC / nct);
                 const int hb = h / a.Hkv, hg = h - hb * a.Hkv;
                 // Columns j0 .. j1-1: warp (gi, quarter) takes j0 + 4 gi + quarter, then
-                // every 8th. Lane k holds the (m, l) of the slab's k-th CTA partial (32 a
-                // round), so the weights take one round of loads; then each lane covers 4
-                // dims and loads 8 partials' o at a time.
+                // every 8th. Per round of 32 partials, lane k loads the k-th partial's
+                // (m, l) once (the weights of the round, with a running rescale when a
+                // slab has more than 32 CTAs); then each lane covers 4 dims and keeps 16
+                // partials' o in flight, so a round costs two or three L2 round trips.
                 const int ncta = c1 - c0 + 1;
                 for (int j = j0 + 4 * gi + quarter; j < j1; j += 8) {
-                    float M = -INFINITY;
-                    for (int k0 = 0; k0 < ncta; k0 += 32) {
-                        const int cc = c0 + k0 + lane;
-                        if (cc <= c1 && (all_live || part_start(cc, R, P) < part_start(cc + 1, R, P)))
-                            M = fmaxf(M, __ldcg(a.work_ml + (((int64_t)cc + h) * NC + j) * 2));
-                    }
-#pragma unroll
-                    for (int o = 16; o >= 1; o >>= 1) M = fmaxf(M, __shfl_xor_sync(kFull, M, o));
-                    float L = 0.f;
+                    float M = -INFINITY, L = 0.f;  // L: this lane's share of the sum
                     float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
                     for (int k0 = 0; k0 < ncta; k0 += 32) {
                         const int cc = c0 + k0 + lane;
                         const bool okp = cc <= c1 && (all_live || part_start(cc, R, P) < part_start(cc + 1, R, P));
                         const float2 ml = okp ? __ldcg(reinterpret_cast<const float2*>(a.work_ml + (((int64_t)cc + h) * NC + j) * 2))
                                               : make_float2(-INFINITY, 0.f);
-                        const float f = (ml.x == -INFINITY) ? 0.f : ex2(ml.x - M);
-                        L = fmaf(ml.y, f, L);
-                        const int n = min(32, ncta - k0);
-                        for (int u0 = 0; u0 < n; u0 += 8) {
-                            float4 v[8];
-                            float fk[8];
+                        float rm = ml.x;
 #pragma unroll
-                            for (int u = 0; u < 8; ++u) {
+                        for (int o = 16; o >= 1; o >>= 1) rm = fmaxf(rm, __shfl_xor_sync(kFull, rm, o));
+                        const float Mn = fmaxf(M, rm);
+                        const float sc = M == -INFINITY ? 0.f : ex2(M - Mn);  // rescale of the earlier rounds
+                        const float f = ml.x == -INFINITY ? 0.f : ex2(ml.x - Mn);
+                        M = Mn;
+                        L = fmaf(ml.y, f, L * sc);
+                        O.x *= sc;
+                        O.y *= sc;
+                        O.z *= sc;
+                        O.w *= sc;
+                        const int n = min(32, ncta - k0);
+                        for (int u0 = 0; u0 < n; u0 += 16) {
+                            float4 v[16];
+                            float fk[16];
+#pragma unroll
+                            for (int u = 0; u < 16; ++u) {
                                 const int k = u0 + u;
                                 fk[u] = __shfl_sync(kFull, f, k & 31);
                                 const bool okk = __shfl_sync(kFull, okp ? 1 : 0, k & 31) != 0 && k < n;
@@ -926,7 +935,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                                 if (!okk) fk[u] = 0.f;
                             }
 #pragma unroll
-                            for (int u = 0; u < 8; ++u) {
+                            for (int u = 0; u < 16; ++u) {
                                 O.x = fmaf(v[u].x, fk[u], O.x);
                                 O.y = fmaf(v[u].y, fk[u], O.y);
                                 O.z = fmaf(v[u].z, fk[u], O.z);
