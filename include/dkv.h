@@ -60,6 +60,7 @@ typedef enum {
 #define DKV_DEV_APPEND_OVERFLOW 0x1 /* n_appended reached the slab's reserve: token not appended */
 #define DKV_DEV_TMA_TIMEOUT 0x2     /* a bulk copy did not complete within the wait bound */
 #define DKV_DEV_MERGE_TIMEOUT 0x4   /* a fused merge's partials were not all written within the wait bound */
+#define DKV_DEV_BOUNDS 0x8          /* bounds-checked build only: an index or offset a kernel read was out of its range; the access was skipped */
 
 /* Pattern and model geometry (Sec. 3.2, Sec. 3.4). */
 typedef struct {

@@ -342,6 +342,7 @@ static dkv_status map_pattern_impl(const uint8_t* M_host, const int32_t* ctx_len
     ma.reserve = reserve_rows;
     ma.NH = NH;
     ma.stride = inplace_stride;
+    ma.status = p->d_status;
     if ((st = launched(dkv::launch_map(ma, stream), "map kernels")) != DKV_OK) return bail(st);
     // The one synchronisation: the totals (rows, kept rows, longest slab, rows of each layer).
     std::vector<int64_t> tail((size_t)3 + s->L);
@@ -506,6 +507,8 @@ dkv_status dkv_compact_inplace(const dkv_plan* p, void* K, void* V, cudaStream_t
     a.T_stride = p->inplace_stride;
     a.kept = p->kept_rows;
     a.NH = p->s.L * p->B * p->s.H_kv;
+    a.status = p->d_status;
+    a.rows_cap = (int64_t)a.NH * p->inplace_stride;
     dkv_status st =
         launched(dkv::launch_compact_inplace(a, p->d_order, p->d_order + a.NH, stream), "in-place compact kernel");
     return st == DKV_OK ? ok() : st;
@@ -557,6 +560,8 @@ dkv_status dkv_compact(const dkv_plan* p, const void* K, const void* V, int64_t 
     a.T_stride = T_stride;
     a.kept = p->kept_rows;
     a.NH = p->s.L * p->B * p->s.H_kv;
+    a.status = p->d_status;
+    a.rows_cap = p->total_rows;
     dkv_status st = launched(dkv::launch_compact(a, stream), "compact kernel");
     return st == DKV_OK ? ok() : st;
 }
@@ -612,6 +617,7 @@ dkv_status decode_args(const dkv_plan* p, int32_t layer, const void* q, const vo
     a->slab_count = p->d_slab_count;
     a->merge_extra = fault("merge") ? 1 : 0;
     a->status = p->d_status;
+    a->rows_cap = p->total_rows;
     a->B = p->B;
     a->H = p->s.H;
     a->Hkv = p->s.H_kv;

@@ -63,10 +63,14 @@ __global__ void __launch_bounds__(kThreads) compact_kernel(const CompactArgs a)
         if (row < a.kept) {
             int hr = h;
             while (a.ioff[hr + 1] <= row) ++hr;
-            const int64_t src = (int64_t)hr * a.T_stride + a.idx[row];
-            dst[i] = a.off[hr] + (row - a.ioff[hr]);
-            kv[i] = ld_stream(reinterpret_cast<const uint4*>(a.K + src * kHeadDim) + sub);
-            vv[i] = ld_stream(reinterpret_cast<const uint4*>(a.V + src * kHeadDim) + sub);
+            const int32_t ix = a.idx[row];
+            const int64_t d = a.off[hr] + (row - a.ioff[hr]);
+            if (in_bounds(ix >= 0 && ix < a.T_stride && d >= 0 && d < a.rows_cap, a.status)) {
+                const int64_t src = (int64_t)hr * a.T_stride + ix;
+                dst[i] = d;
+                kv[i] = ld_stream(reinterpret_cast<const uint4*>(a.K + src * kHeadDim) + sub);
+                vv[i] = ld_stream(reinterpret_cast<const uint4*>(a.V + src * kHeadDim) + sub);
+            }
         }
     }
 #pragma unroll
@@ -169,6 +173,10 @@ __global__ void __launch_bounds__(kIpThreads, 1)
 #pragma unroll
             for (int i = 0; i < kIpPer; ++i) {
                 cur[i] = nxt[i];
+                // A row only moves towards its slab's start, inside the slab's region.
+                if (cur[i] >= 0 &&
+                    !in_bounds(cur[i] >= r0 + warp + kIpWarps * i && cur[i] < a.T_stride, a.status))
+                    cur[i] = -1;
                 if (cur[i] >= 0) {
                     const uint16_t* src = (kv ? V : K) + (base + cur[i]) * kHeadDim;
                     v[i] = __ldcg(reinterpret_cast<const uint4*>(src) + c);

@@ -384,7 +384,11 @@ __global__ void __launch_bounds__(C::NW * 32, 1) decode_partial_kernel(const Dec
         auto issue = [&](const Cursor& cu, int stage) {
             const int cnt = min(TR, cu.s1 - cu.x);
             const int r0 = cu.x - cu.p0;  // row within the slab
-            const int ncopy = (cu.app && r0 + cnt == cu.n_h) ? cnt - 1 : cnt;  // new token comes from k_new
+            int ncopy = (cu.app && r0 + cnt == cu.n_h) ? cnt - 1 : cnt;  // new token comes from k_new
+            // Bounds-checked build: rows outside the cache are not copied (the stage's
+            // barrier then expects no bytes, so its wait still completes).
+            if (!in_bounds(cu.base + r0 >= 0 && (a.rows_cap == 0 || cu.base + r0 + ncopy <= a.rows_cap), a.status))
+                ncopy = 0;
             const uint32_t bar = smem_u32(&my_bars[stage]);
             unsigned char* dst = my_ring + stage * C::kStageBytes;
             const uint32_t bytes = (uint32_t)ncopy * kRowBytes;
@@ -475,8 +479,11 @@ __global__ void __launch_bounds__(C::NW * 32, 1) decode_partial_kernel(const Dec
                     const uint16_t* src = (half ? a.v_new : a.k_new) + ((int64_t)b * a.Hkv + g) * kHeadDim;
                     const uint4 v = __ldg(reinterpret_cast<const uint4*>(src) + sub);
                     *reinterpret_cast<uint4*>((half ? vt : kt) + (cnt - 1) * kRowBytes + sub * 16) = v;
-                    uint16_t* dstg = (half ? a.Vc : a.Kc) + (cp.base + (cp.n_h - 1)) * kHeadDim;
-                    *(reinterpret_cast<uint4*>(dstg) + sub) = v;
+                    const int64_t nrow = cp.base + (cp.n_h - 1);
+                    if (in_bounds(nrow >= 0 && (a.rows_cap == 0 || nrow < a.rows_cap), a.status)) {
+                        uint16_t* dstg = (half ? a.Vc : a.Kc) + nrow * kHeadDim;
+                        *(reinterpret_cast<uint4*>(dstg) + sub) = v;
+                    }
                     fence_proxy_async_smem();  // order these generic writes before later bulk copies
                     __syncwarp();
                 }

@@ -407,6 +407,9 @@ __global__ void __launch_bounds__(MKFor<G, NT, MULTI>::NW * 32, 1)
         // overwritten in shared memory from k_new / v_new.)
         auto issue = [&](const Cursor& cu, int stage) {
             const int row = (int)(cu.base + (cu.x - cu.p0));
+            // Bounds-checked build: the tile's rows lie in the cache (a TMA box past
+            // the end reads zeros, so the copy itself stays in bounds either way).
+            in_bounds(row >= 0 && (a.rows_cap == 0 || row + min(C::TR, cu.s1 - cu.x) <= a.rows_cap), a.status);
             const uint32_t bar = smem_u32(&my_bars[stage]);
             const uint32_t dst = smem_u32(my_ring + stage * C::kStageBytes);
             fence_proxy_async_smem();
@@ -478,8 +481,11 @@ __global__ void __launch_bounds__(MKFor<G, NT, MULTI>::NW * 32, 1)
                     const uint16_t* src = (kv ? a.v_new : a.k_new) + ((int64_t)b * a.Hkv + g) * kHeadDim;
                     const uint4 v = __ldg(reinterpret_cast<const uint4*>(src) + sub);
                     *reinterpret_cast<uint4*>(st + (2 * kv + (sub >> 3)) * kBoxBytes + swz(cnt - 1, sub & 7)) = v;
-                    uint16_t* dstg = (kv ? a.Vc : a.Kc) + (cp.base + (cp.n_h - 1)) * kHeadDim;
-                    *(reinterpret_cast<uint4*>(dstg) + sub) = v;
+                    const int64_t nrow = cp.base + (cp.n_h - 1);
+                    if (in_bounds(nrow >= 0 && (a.rows_cap == 0 || nrow < a.rows_cap), a.status)) {
+                        uint16_t* dstg = (kv ? a.Vc : a.Kc) + nrow * kHeadDim;
+                        *(reinterpret_cast<uint4*>(dstg) + sub) = v;
+                    }
                     touched = true;
                 }
                 if (cnt < TR) {

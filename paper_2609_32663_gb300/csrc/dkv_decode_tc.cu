@@ -425,6 +425,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         waited = true;
                     }
                     const int s = tk % kKStages, row = wk.cache_row();
+                    // Bounds-checked build: the tile's rows lie in the cache (TMA reads
+                    // zeros past the end, so the copy stays in bounds either way).
+                    in_bounds(row >= 0 && (a.rows_cap == 0 || row + wk.cnt() <= a.rows_cap), a.status);
                     const uint32_t bar = smem_u32(&k_full[s]), dst = smem_u32(ringK + s * kTcHalfTile);
                     mbar_arrive_expect_tx(bar, kTcHalfTile);
 #pragma unroll

@@ -11,6 +11,21 @@ namespace dkv {
 constexpr int kHeadDim = 128;   // elements per row
 constexpr int kRowBytes = 256;  // bytes per bf16 row
 
+// Bounds-checked build (-DDKV_DEBUG, build.build_library(debug=True)): the
+// kernels check the indices and offsets they read against the ranges the plan
+// gives them, skip an access that falls outside, and set DKV_DEV_BOUNDS in the
+// plan's status word. No trap and no assert, so the context stays usable and
+// the host reads the word. In the normal build the checks compile to nothing.
+#ifdef DKV_DEBUG
+__device__ __forceinline__ bool in_bounds(bool ok, int32_t* status)
+{
+    if (!ok && status) atomicOr(status, 0x8 /* DKV_DEV_BOUNDS */);
+    return ok;
+}
+#else
+__device__ __forceinline__ constexpr bool in_bounds(bool, int32_t*) { return true; }
+#endif
+
 // ---------------------------------------------------------------- pattern map
 struct MapArgs {
     const uint8_t* M;       // [L][H][D]
@@ -27,6 +42,7 @@ struct MapArgs {
     int L, H, Hkv, D, B, sink, recent, bin_width, reserve;
     int NH;                 // L*B*Hkv
     int64_t stride;         // 0: slabs packed end to end; > 0: slab h starts at row h * stride (in place)
+    int32_t* status;        // the plan's device status word (bounds-checked build)
 };
 constexpr int kMapChunk = 8192;  // output rows per CTA of the index-list write
 
@@ -49,6 +65,8 @@ struct CompactArgs {
     int64_t T_stride;
     int64_t kept;
     int NH;
+    int32_t* status;        // the plan's device status word (bounds-checked build)
+    int64_t rows_cap;       // rows of the packed cache (out of place) or of each buffer (in place)
 };
 cudaError_t launch_compact(const CompactArgs& a, cudaStream_t st);
 // In place: K and V are both source and destination, slab h at rows h * T_stride
@@ -74,6 +92,7 @@ struct DecodeArgs {
     float* out;             // [B][H][128]
     int32_t* slab_count;    // [B*Hkv][cols][2] arrivals, partials written (zero between calls)
     int32_t* status;
+    int64_t rows_cap;       // rows of Kc/Vc, for the bounds-checked build; 0 when the caller does not give it
     int B, H, Hkv, G;
     int reserve;
     int append;             // 1 when k_new/v_new are given

@@ -202,6 +202,10 @@ __global__ void __launch_bounds__(kWriteThreads) write_kernel(const MapArgs a)
     __syncthreads();
     const int2* run = staged ? srun : grun;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // Bounds-checked build: the slab's indices lie inside the list, and every
+    // position inside its sequence's context (checked per row below).
+    const int Tcb = __ldg(a.Tc + (h / a.Hkv) % a.B);
+    if (!in_bounds(__ldg(a.ioff + h) + n_h <= __ldg(a.ioff + a.NH), a.status)) return;  // uniform
     int32_t* dst = a.idx + __ldg(a.ioff + h);
     // Lane rows: base + 32 k, k < 32 (the warp covers 1024 consecutive rows).
     const int base = r0 + warp * (kMapChunk / (kWriteThreads / 32)) + lane;
@@ -227,7 +231,8 @@ __global__ void __launch_bounds__(kWriteThreads) write_kernel(const MapArgs a)
             cur = run[i];
             next = i + 1 < nr ? run[i + 1].x : n_h;
         }
-        dst[r] = cur.y + (r - cur.x);
+        const int pos = cur.y + (r - cur.x);
+        if (in_bounds(pos >= 0 && pos < Tcb, a.status)) dst[r] = pos;
     }
 }
 

@@ -16,12 +16,15 @@ from dataclasses import dataclass
 import numpy as np
 
 _PKG = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_PKG, "libdkv.so")
+# DKV_LIBRARY names another build of the same ABI to load instead, e.g. the
+# bounds-checked libdkv_debug.so (build.build_library(debug=True)).
+LIB_PATH = os.environ.get("DKV_LIBRARY") or os.path.join(_PKG, "libdkv.so")
 
 DKV_OK, DKV_ERR_INVALID_ARG, DKV_ERR_CUDA, DKV_ERR_OOM, DKV_ERR_RANGE, DKV_ERR_TIMEOUT = range(6)
 DKV_DEV_APPEND_OVERFLOW = 0x1
 DKV_DEV_TMA_TIMEOUT = 0x2
 DKV_DEV_MERGE_TIMEOUT = 0x4
+DKV_DEV_BOUNDS = 0x8
 
 # Every entry point include/dkv.h declares.
 EXPORTS = ("dkv_last_error", "dkv_map_pattern", "dkv_plan_dense", "dkv_plan_query", "dkv_plan_read",

@@ -10,6 +10,9 @@ import oracle as O
 import paper_2609_32663_gb300.dkv as dkv
 from paper_2609_32663_gb300 import inputs as I
 
+# True when the tests run against the bounds-checked build (DKV_LIBRARY=.../libdkv_debug.so).
+BOUNDS_CHECKED = os.environ.get("DKV_LIBRARY", "").endswith("libdkv_debug.so")
+
 # Tolerances of the fp32 attention output against the fp64 oracle.
 REL_L2 = 1e-3
 MAX_ABS = 5e-3
@@ -138,4 +141,8 @@ class Case:
                 f"slab {h} bytes differ after appends"
 
     def close(self):
+        # Under the bounds-checked build every case also asserts that no kernel
+        # flagged an out-of-range index or offset.
+        word = dkv.dkv_plan_status(self.plan) if BOUNDS_CHECKED else 0
         self.plan.close()
+        assert not word & dkv.DKV_DEV_BOUNDS, f"bounds-checked build flagged an access (status {word:#x})"

@@ -245,3 +245,12 @@ def test_header_is_plain_c_and_links_from_c(dkvmod, tmp_path):
                            "-L", libdir, "-ldkv", f"-Wl,-rpath,{libdir}"])
     out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout
     assert int(out) == len(names)
+
+
+def test_bounds_checked_build_exports_every_declared_symbol(dkvmod):
+    """The -DDKV_DEBUG variant (libdkv_debug.so) compiles from the same sources
+    and exports the same ABI; its kernels run in tests/test_gpu_bounds_build.py."""
+    from paper_2609_32663_gb300 import build
+    lib = ctypes.CDLL(build.build_library(debug=True))
+    for name in declared_functions():
+        assert hasattr(lib, name), name
