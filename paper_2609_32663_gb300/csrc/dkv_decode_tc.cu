@@ -77,6 +77,7 @@ constexpr int kTcQHalf = kTcQRows * 128;       // one 64-dim half of Q (8 KB)
 constexpr int kTcQBytes = 2 * kTcQHalf;        // Q as the A operand: 64 rows x 128 dims (two buffers: segments alternate)
 constexpr int kTcPBytes = 2 * kTcMaxCols * 128;  // one P buffer: high parts (rows 0..NCpad-1), then low parts, 64 rows each
 constexpr int kSBufs = 4;                      // TMEM score buffers
+static_assert((kKStages & (kKStages - 1)) == 0 && (kSBufs & (kSBufs - 1)) == 0, "indexed by masks");
 constexpr int kTcTmemCols = 512;               // S buffers at columns 0, 64, 128, 192; O of group g at 256 + 128 g
 constexpr int kTcOCols = 2 * kTcMaxCols;       // O of one group: the product with P's high parts, then with its low parts
 constexpr int kTcOCol = kSBufs * kTcRows;
@@ -503,18 +504,22 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         if (lane == 0) {
             const uint32_t id1 = idesc(kTcQRows, kTcRows, 0, 0);
             const uint32_t id2 = idesc(128, 2 * NCpad, 1, 0);  // high and low parts of P side by side
-            // Operand descriptors of the first stage of each ring; a stage or k-step
-            // further on is a constant added to the address field (16-byte units; every
-            // shared-memory address is below 2^18 bytes, so the 14-bit field never
-            // carries). One thread issues every product, so its per-product work is the
-            // pipeline's pace: nothing is recomputed per k-step.
-            const uint64_t dQ = sdesc(smem_u32(sQ), 16, 1024);
-            const uint64_t dK = sdesc(smem_u32(ringK), 16, 1024);
-            const uint64_t dV = sdesc(smem_u32(ringV), kTcBox, 1024);
-            const uint64_t dP = sdesc(smem_u32(sP), 16, 1024);
+            // Operand descriptors: every operand here has a stride byte offset of 1 KB,
+            // version 1 and the 128-byte swizzle, so the high word is one constant; a
+            // stage or k-step further on adds to the address field of the low word (16-byte
+            // units; every shared-memory address is below 2^18 bytes, so the 14-bit field
+            // never carries). One thread issues every product and its per-product work is
+            // the pipeline's pace, so the loop keeps to 32-bit adds and running counters.
+            const uint32_t dhi = (uint32_t)(sdesc(0, 0, 1024) >> 32);
+            const uint32_t dQ = (uint32_t)sdesc(smem_u32(sQ), 16, 1024);
+            const uint32_t dK = (uint32_t)sdesc(smem_u32(ringK), 16, 1024);
+            const uint32_t dV = (uint32_t)sdesc(smem_u32(ringV), kTcBox, 1024);
+            const uint32_t dP = (uint32_t)sdesc(smem_u32(sP), 16, 1024);
+            auto desc = [dhi](uint32_t lo) { return ((uint64_t)dhi << 32) | lo; };
             TileWalk w1;
             w1.begin(a, tab, hfirst, hend, A, Bc);
             int t1 = 0, t2 = 0, seg = 0, seg_start = 0;
+            int vs = 0;  // V stage of tile t2 (t2 % kVStages)
             // Bit t % kSBufs: tile t (between the two products) is one of the first two
             // of its segment, so its group's output product starts the accumulator afresh.
             uint32_t fresh_bits = 0;
@@ -524,30 +529,32 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             while (w1.more() || t2 < t1) {
                 bool moved = false;
                 // Output products first: the softmax group of tile t2 waits for it before
-                // it can write its next P.
+                // it can write its next P. P of a tile is announced only after its V stage
+                // landed (the group's leader waits for it), so p_full is the one test.
                 if (t2 < t1) {
-                    const int b = t2 & 1, s = t2 % kVStages;
-                    if (test_phase(&p_full[b], (t2 >> 1) & 1) && test_phase(&v_full[s], (t2 / kVStages) & 1)) {
+                    const int b = t2 & 1;
+                    if (test_phase(&p_full[b], (t2 >> 1) & 1)) {
                         tc_fence_after();
                         // O^T += V^T [P_hi P_lo] into the group's accumulator (the two
                         // halves are summed when O is read); a group's first tile of a
                         // segment starts it afresh.
-                        const uint64_t va = dV + (uint64_t)(s * (kTcHalfTile >> 4));
-                        const uint64_t pb = dP + (uint64_t)(b * (kTcPBytes >> 4));
+                        const uint32_t va = dV + (uint32_t)vs * (kTcHalfTile >> 4);
+                        const uint32_t pb = dP + (uint32_t)b * (kTcPBytes >> 4);
                         const uint32_t o = tmem + kTcOCol + b * kTcOCols;
-                        const uint32_t fresh = (fresh_bits >> (t2 % kSBufs)) & 1u;
-                        umma(o, va, pb, id2, fresh ^ 1u);
+                        const uint32_t fresh = (fresh_bits >> (t2 & (kSBufs - 1))) & 1u;
+                        umma(o, desc(va), desc(pb), id2, fresh ^ 1u);
 #pragma unroll
                         for (int k = 1; k < kTcRows / 16; ++k)
-                            umma(o, va + (uint64_t)(k * (2048 >> 4)), pb + (uint64_t)(k * (32 >> 4)), id2, 1u);
+                            umma(o, desc(va + k * (2048 >> 4)), desc(pb + k * (32 >> 4)), id2, 1u);
                         umma_commit(smem_u32(&o_done[b]));
-                        umma_commit(smem_u32(&v_empty[s]));
+                        umma_commit(smem_u32(&v_empty[vs]));
                         ++t2;
+                        if (++vs == kVStages) vs = 0;
                         moved = true;
                     }
                 }
                 if (w1.more() && t1 < t2 + kSBufs) {
-                    const int s = t1 % kKStages;
+                    const int s = t1 & (kKStages - 1);
                     const bool first = w1.first();
                     if (first && !qseen && test_phase(&q_full[seg & 1], (seg >> 1) & 1)) {
                         qbuf = seg & 1;
@@ -559,16 +566,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         tc_fence_after();
                         // S^T[64 x 64] = Q[64 x 128] K^T: k-steps of 16 dims (+32 B inside a
                         // 64-dim half, +kTcBox or +kTcQHalf to the next half).
-                        const uint64_t qa = dQ + (uint64_t)(qbuf * (kTcQBytes >> 4));
-                        const uint64_t kb = dK + (uint64_t)(s * (kTcHalfTile >> 4));
-                        const uint32_t d = tmem + (t1 % kSBufs) * kTcRows;
+                        const uint32_t qa = dQ + (uint32_t)qbuf * (kTcQBytes >> 4);
+                        const uint32_t kb = dK + (uint32_t)s * (kTcHalfTile >> 4);
+                        const uint32_t d = tmem + (t1 & (kSBufs - 1)) * kTcRows;
 #pragma unroll
                         for (int k = 0; k < 8; ++k)
-                            umma(d, qa + (uint64_t)((k >> 2) * (kTcQHalf >> 4) + (k & 3) * 2),
-                                 kb + (uint64_t)((k >> 2) * (kTcBox >> 4) + (k & 3) * 2), id1, k > 0 ? 1u : 0u);
-                        umma_commit(smem_u32(&s_full[t1 % kSBufs]));
+                            umma(d, desc(qa + (k >> 2) * (kTcQHalf >> 4) + (k & 3) * 2),
+                                 desc(kb + (k >> 2) * (kTcBox >> 4) + (k & 3) * 2), id1, k > 0 ? 1u : 0u);
+                        umma_commit(smem_u32(&s_full[t1 & (kSBufs - 1)]));
                         umma_commit(smem_u32(&k_empty[s]));
-                        const uint32_t bit = 1u << (t1 % kSBufs);
+                        const uint32_t bit = 1u << (t1 & (kSBufs - 1));
                         fresh_bits = (t1 - seg_start < 2) ? (fresh_bits | bit) : (fresh_bits & ~bit);
                         issued = true;
                         qseen = false;
@@ -637,7 +644,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 if (gleader) {
                     bool ok = !flags[kFlagAbort] && wait_phase(&s_full[t % kSBufs], (t / kSBufs) & 1);
                     if (ok && gfirst && t >= 2) ok = wait_phase(&o_done[b], ((t - 2) >> 1) & 1);
-                    if (ok && cnt < kTcRows) ok = wait_phase(&v_full[t % kVStages], (t / kVStages) & 1);
+                    // The tile's V stage (zeroed below past a partial tile's rows; and P is
+                    // announced to the MMA lane only once V has landed).
+                    if (ok) ok = wait_phase(&v_full[t % kVStages], (t / kVStages) & 1);
                     if (!ok && !flags[kFlagAbort]) {
                         atomicOr(a.status, kDevTmaTimeout);
                         flags[kFlagAbort] = 1;
