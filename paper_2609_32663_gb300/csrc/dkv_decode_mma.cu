@@ -71,6 +71,19 @@ struct MK {
 #ifndef DKV_MMA_CFG_MULTI
 #define DKV_MMA_CFG_MULTI 2, 12
 #endif
+// Right after the wait for the previous kernel, a warp has one tile landed and
+// one in flight: half its ring. The rows of its next kL2Tiles tiles are
+// prefetched into L2 then, to fill the memory pipe while its first tiles are
+// computed. Measured (same-box A/B, us per step): llama8b-128k 1,091 -> 1,069
+// with 2 tiles (1,081 with 4); qwen7b-64k-b4-r20 716 -> 712. A warp with a short
+// range gains nothing and its prefetches delay the copies its first tiles wait
+// for: prefetching at llama8b-32k (3-4 tiles a warp) took 466 -> 516, so only
+// warps with at least kL2MinRows rows prefetch (32K: 469 -> 471, none do). The
+// same prefetches issued before the wait competed with the previous kernel's
+// end-of-pass merge and measured slower at every size.
+constexpr int kL2Tiles = 2;
+constexpr int kL2MinRows = 64;
+
 template <int G, int NT, bool MULTI>
 using MKFor = typename std::conditional<
     (NT > 1), MK<G, NT, DKV_MMA_CFG_MULTI>,
@@ -449,6 +462,17 @@ __global__ void __launch_bounds__(MKFor<G, NT, MULTI>::NW * 32, 1)
         for (int s = PRE; s < NS && ld.h < hend; ++s) {
             ++inflight;
             cursor_next<TR>(ld, a, tab, hend, wA, wB);
+        }
+        if (lane == 0 && wB - wA >= kL2MinRows) {
+            // The next tiles' K and V rows into L2: exactly the segment's rows, all in the cache.
+            Cursor it = ld;
+            for (int s = 0; s < kL2Tiles && it.h < hend; ++s) {
+                const int cnt = min(TR, it.s1 - it.x);
+                const int64_t row = it.base + (it.x - it.p0);
+                prefetch_l2_bulk(a.Kc + row * kHeadDim, (uint32_t)cnt * kRowBytes);
+                prefetch_l2_bulk(a.Vc + row * kHeadDim, (uint32_t)cnt * kRowBytes);
+                cursor_next<TR>(it, a, tab, hend, wA, wB);
+            }
         }
         int stage = 0;
         uint32_t phase = 0;
