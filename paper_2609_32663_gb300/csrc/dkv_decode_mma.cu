@@ -75,13 +75,14 @@ struct MK {
 // one in flight: half its ring. The rows of its next kL2Tiles tiles are
 // prefetched into L2 then, to fill the memory pipe while its first tiles are
 // computed. Measured (same-box A/B, us per step): llama8b-128k 1,091 -> 1,069
-// with 2 tiles (1,081 with 4); qwen7b-64k-b4-r20 716 -> 712. A warp with a short
-// range gains nothing and its prefetches delay the copies its first tiles wait
-// for: prefetching at llama8b-32k (3-4 tiles a warp) took 466 -> 516, so only
-// warps with at least kL2MinRows rows prefetch (32K: 469 -> 471, none do). The
-// same prefetches issued before the wait competed with the previous kernel's
+// with 1 or 2 tiles (1,076 with 3, 1,081 with 4); qwen7b-64k-b4-r20 716 -> 712;
+// qwen7b-64k-b4-r50 1,285 with 2 tiles, 1,277 with 1. A warp with a short range
+// gains nothing and its prefetches delay the copies its first tiles wait for:
+// prefetching at llama8b-32k (3-4 tiles a warp) took 466 -> 516, so only warps
+// with at least kL2MinRows rows prefetch (32K: 469 -> 471, none do). The same
+// prefetches issued before the wait competed with the previous kernel's
 // end-of-pass merge and measured slower at every size.
-constexpr int kL2Tiles = 2;
+constexpr int kL2Tiles = 1;
 constexpr int kL2MinRows = 64;
 
 template <int G, int NT, bool MULTI>
