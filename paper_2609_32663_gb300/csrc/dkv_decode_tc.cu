@@ -343,6 +343,69 @@ struct IdleBound {
     }
 };
 
+// Row partition of a layer over the CTAs. A CTA whose range holds a slab
+// boundary drains its pipeline at that segment's end (~5 us), and the slab's
+// merge waits for it. So while the slabs are few (at most a quarter as many as
+// the CTAs) and the rounding keeps every CTA within 1.15 shares of rows, each
+// slab gets a whole number of CTAs, cb(h+1) - cb(h) with cb(h) = round(P S_h / R)
+// (S_h: the slab's first row), and splits its rows evenly over them. An empty
+// slab gets no CTA and lies inside the CTA that starts the next one. Otherwise
+// the rows are cut into P equal ranges, as in the other decode kernels. Every
+// CTA evaluates the same float expressions, so all agree on the partition.
+struct TcPart {
+    bool aligned;
+    int R, P, NHl;
+    float scale;  // P / R
+    __device__ int cb(const DecodeArgs& a, const SeqTable& t, int h) const
+    {
+        if (h >= NHl) return P;
+        return min(P, (int)floorf(fmaf((float)slab_start(a, t, h), scale, 0.5f)));
+    }
+    // First row of CTA c (c <= P).
+    __device__ int start(const DecodeArgs& a, const SeqTable& t, int c) const
+    {
+        if (!aligned) return part_start(c, R, P);
+        if (c >= P) return R;
+        int lo = 0, hi = NHl - 1;  // home slab: the first h with cb(h + 1) > c
+        while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (cb(a, t, mid + 1) > c)
+                hi = mid;
+            else
+                lo = mid + 1;
+        }
+        const int f = lo, cf = cb(a, t, f);
+        if (c == cf) {  // the first CTA of slab f also takes the slabs before it that got no CTA
+            int l2 = 0, h2 = f;
+            while (l2 < h2) {
+                const int mid = (l2 + h2) >> 1;
+                if (cb(a, t, mid) >= c)
+                    h2 = mid;
+                else
+                    l2 = mid + 1;
+            }
+            return slab_start(a, t, l2);
+        }
+        const int s0 = slab_start(a, t, f);
+        const unsigned nf = (unsigned)(slab_start(a, t, f + 1) - s0), n = (unsigned)(cb(a, t, f + 1) - cf);
+        const unsigned w = (unsigned)(c - cf), q = nf / n, r = nf - q * n;  // floor(w nf / n), w r < n^2
+        return s0 + (int)(w * q + (w * r) / n);
+    }
+    // CTAs whose ranges overlap slab h (with rows [p0, p1)): their count, first and last.
+    __device__ int slab_ctas(const DecodeArgs& a, const SeqTable& t, int h, int p0, int p1, int* c0, int* c1) const
+    {
+        if (!aligned) return ctas_of_slab(p0, p1, R, P, c0, c1);
+        const int b0 = cb(a, t, h), b1 = cb(a, t, h + 1);
+        if (b1 > b0) {
+            *c0 = b0;
+            *c1 = b1 - 1;
+            return b1 - b0;
+        }
+        *c0 = *c1 = min(b0, P - 1);
+        return 1;
+    }
+};
+
 template <int G>
 __global__ void __launch_bounds__(kTcThreads, 1)
     decode_tc_kernel(const __grid_constant__ DecodeArgs a, const __grid_constant__ CacheMaps maps)
@@ -397,7 +460,20 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 for (int j = 0; j < a.NC; ++j)
                     write_out<G>(a, h / a.Hkv, h % a.Hkv, j, make_float4(0.f, 0.f, 0.f, 0.f), 0.f, lane);
     }
-    const int A = part_start(c, R, a.nctas), Bc = part_start(c + 1, R, a.nctas);
+    TcPart part;
+    part.R = R;
+    part.P = a.nctas;
+    part.NHl = NHl;
+    part.scale = (float)a.nctas / (float)max(R, 1);
+    part.aligned = NHl * 4 <= a.nctas && R >= 4 * a.nctas;
+    // Only while no CTA would get more than 1.15 shares of rows (R / P), and every
+    // slab with rows gets a CTA of its own.
+    for (int h = 0; h < NHl && part.aligned; ++h) {
+        const int rows = slab_start(a, tab, h + 1) - slab_start(a, tab, h);
+        const int n = part.cb(a, tab, h + 1) - part.cb(a, tab, h);
+        if (rows > 0 && (n < 1 || (float)rows * part.scale > 1.15f * (float)n)) part.aligned = false;
+    }
+    const int A = part.start(a, tab, c), Bc = part.start(a, tab, c + 1);
     if (A >= Bc) return;  // uniform: this CTA has no rows (no TMEM taken yet)
     const int hfirst = slab_containing(a, tab, NHl, A);
     const int hend = slab_containing(a, tab, NHl, Bc - 1) + 1;
@@ -869,7 +945,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             if (e == 1 && h == hfirst) break;
             const int p0 = slab_start(a, tab, h), p1 = slab_start(a, tab, h + 1);
             int c0 = 0, c1 = 0;
-            const int nct = ctas_of_slab(p0, p1, R, P, &c0, &c1);
+            const int nct = part.slab_ctas(a, tab, h, p0, p1, &c0, &c1);
             if (nct <= 1) continue;  // uniform: written at its segment's end
             int32_t* ctr = a.slab_count + (int64_t)h * kMaxCols * 2;
             if (leader) {
@@ -901,7 +977,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 if (all_live) {
                     k = c - c0;
                 } else {
-                    for (int cc = c0; cc < c; ++cc) k += part_start(cc, R, P) < part_start(cc + 1, R, P) ? 1 : 0;
+                    for (int cc = c0; cc < c; ++cc) k += part.start(a, tab, cc) < part.start(a, tab, cc + 1) ? 1 : 0;
                 }
                 const int j0 = (int)((int64_t)k * NC / nct), j1 = (int)((int64_t)(k + 1) * NC / nct);
                 const int hb = h / a.Hkv, hg = h - hb * a.Hkv;
@@ -916,7 +992,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
                     for (int k0 = 0; k0 < ncta; k0 += 32) {
                         const int cc = c0 + k0 + lane;
-                        const bool okp = cc <= c1 && (all_live || part_start(cc, R, P) < part_start(cc + 1, R, P));
+                        const bool okp = cc <= c1 && (all_live || part.start(a, tab, cc) < part.start(a, tab, cc + 1));
                         const float2 ml = okp ? __ldcg(reinterpret_cast<const float2*>(a.work_ml + (((int64_t)cc + h) * NC + j) * 2))
                                               : make_float2(-INFINITY, 0.f);
                         float rm = ml.x;

@@ -107,6 +107,44 @@ def test_multi_query_tcgen05_short_and_empty_slabs(Tc):
     case.close()
 
 
+def test_multi_query_tcgen05_slab_aligned_partition(cuda):
+    """Few slabs of uneven lengths, two of them empty: the tcgen05 kernel gives
+    each slab a whole number of CTAs (no CTA range holds a slab boundary) and an
+    empty slab lies inside the CTA that starts the next one. Two layers, with
+    rows appended in an earlier step (the appended rows move every boundary)."""
+    Tc = [30000, 0, 12000, 25000]
+    w = wl(L=2, H=16, Hkv=2, T=max(Tc), B=len(Tc), D=24, W=-(-(30000 - 1152) // 24), ragged=None,
+           outlier_frac=0.01, seed=123)
+    case = Case(w, reserve=4, Tc=np.array(Tc, np.int32))
+    Q = 5  # G = 8: 40 columns
+    gen = torch.Generator().manual_seed(4321)
+    kn = torch.randn((w.L, w.B, w.Hkv, w.head_dim), generator=gen).to(torch.bfloat16)
+    vn = torch.randn((w.L, w.B, w.Hkv, w.head_dim), generator=gen).to(torch.bfloat16)
+    n_app = torch.zeros(w.B, dtype=torch.int32, device=case.dev)
+    na = np.zeros(w.B, np.int32)
+    step_out = torch.empty((w.B, w.H, w.head_dim), dtype=torch.float32, device=case.dev)
+    qs = torch.randn((w.L, w.B, w.H, w.head_dim), generator=gen).to(torch.bfloat16)
+    for layer in range(w.L):
+        dkv.dkv_decode_attn(case.plan, layer, qs[layer].to(case.dev), kn[layer].to(case.dev), vn[layer].to(case.dev),
+                            n_app, case.Kc, case.Vc, step_out)
+        O.append(case.om, layer, w.B, w.Hkv, case.reserve, na, I.bf16_bits(kn[layer]), I.bf16_bits(vn[layer]),
+                 case.oKc, case.oVc)
+    dkv.dkv_advance(case.plan, n_app)
+    na += 1
+    q = multi_q(w, Q, seed=13)
+    out = torch.full((w.B, Q, w.H, w.head_dim), float("nan"), dtype=torch.float32, device=case.dev)
+    for layer in range(w.L):
+        dkv.dkv_decode_multi(case.plan, layer, q[layer].to(case.dev), Q, n_app, case.Kc, case.Vc, out)
+        torch.cuda.synchronize()
+        got = out.double().cpu().numpy()
+        for qi in range(Q):
+            want = O.decode(case.om, layer, w.B, w.H, w.Hkv, I.bf16_bits(q[layer][:, qi]), case.oKc, case.oVc,
+                            n_rows_app=na)
+            assert_close(got[:, qi], want, f"layer {layer} query {qi}")
+    assert dkv.dkv_plan_status(case.plan) == 0
+    case.close()
+
+
 def test_multi_query_tcgen05_twice_in_a_row_and_after_the_decode_step(cuda):
     """The tcgen05 kernel's workspace and slab bounds are reused: two calls in a
     row on different layers, then a decode step, then the multi-query again."""
