@@ -4,10 +4,11 @@
 // (queries x heads of a KV head's group) per slab.
 //
 // Work split: the layer's rows (every slab end to end, plus the rows appended in
-// earlier steps) are cut into equal contiguous CTA ranges (one CTA per SM, a
-// cooperative launch, so every CTA is resident at once), as in the other decode
-// kernels; a CTA walks its range in tiles of 64 rows, slab segment by slab
-// segment (a segment: the part of one slab inside the CTA's range).
+// earlier steps) are cut into contiguous CTA ranges (one CTA per SM, a
+// cooperative launch, so every CTA is resident at once): whole numbers of CTAs
+// per slab while the slabs are few (TcPart below), else equal ranges as in the
+// other decode kernels. A CTA walks its range in tiles of 64 rows, slab segment
+// by slab segment (a segment: the part of one slab inside the CTA's range).
 //
 //   warp 0 (one lane)   TMA: a tile's K rows and V rows, each as 16-row 2-D
 //                       boxes (64 dims, 128-byte swizzle; measured faster than
@@ -24,6 +25,9 @@
 //                       remainder side by side, N = 2 x the columns, one MMA per
 //                       k-step) into the TMEM output accumulator of the tile's
 //                       softmax group, whose two halves are summed when read.
+//                       Output products go first; a group announces its P only
+//                       once the tile's V stage has landed, so that is the one
+//                       barrier the lane tests for them.
 //   warps 2-5, 6-9      two softmax groups; group g takes the tiles t with
 //                       t % 2 == g, with its own running max and sum of every
 //                       column and its own O accumulator (merged at a segment's
@@ -32,9 +36,9 @@
 //                       lanes l and l + 16 of warp (group, quarter) column
 //                       16 quarter + l, rows 0-31 and 32-63 of the tile: tile
 //                       max (one shuffle joins the halves), lazily rescaled
-//                       running max (a column's max
-//                       moves only when a score tops it by kSlack; O is then
-//                       rescaled in TMEM), P = 2^(s - m) written to shared memory
+//                       running max (a column's max moves only when a score
+//                       tops it by kSlackTc; O is then rescaled in TMEM),
+//                       P = 2^(s - m) written to shared memory
 //                       as the B operand of the output product, V rows past a
 //                       segment zeroed. For O, thread (quarter, lane) owns
 //                       dimension 32 quarter + lane (TMEM lane).
