@@ -916,16 +916,20 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         Mv[i] = M;
                         Lv[i] = (has0 ? f0 * g_sum[cc] : 0.f) + (has1 ? f1 * g_sum[kTcMaxCols + cc] : 0.f);
                     }
+                    // Stores that skip L1 (st.global.cg): the L1 path is busy with the
+                    // tiles' shared-memory traffic, and plain stores made a segment's
+                    // end ~2.4 % of the whole launch slower (Q = 8 and 16). Every reader
+                    // of these partials loads them from L2 (ld.global.cg).
 #pragma unroll
                     for (int i = 0; i < 16; ++i) {
                         const int cc = c16 + i;
                         if (cc < NC) {
                             if (whole) {
-                                a.out[out_row<G>(a, bq, g, cc) * kHeadDim + dim] = Lv[i] > 0.f ? ov[i] / Lv[i] : 0.f;
+                                __stcg(a.out + out_row<G>(a, bq, g, cc) * kHeadDim + dim, Lv[i] > 0.f ? ov[i] / Lv[i] : 0.f);
                             } else {
-                                a.work_o[(slot * NC + cc) * kHeadDim + dim] = ov[i];
+                                __stcg(a.work_o + (slot * NC + cc) * kHeadDim + dim, ov[i]);
                                 if (dim == 0)
-                                    *reinterpret_cast<float2*>(a.work_ml + (slot * NC + cc) * 2) = make_float2(Mv[i], Lv[i]);
+                                    __stcg(reinterpret_cast<float2*>(a.work_ml + (slot * NC + cc) * 2), make_float2(Mv[i], Lv[i]));
                             }
                         }
                     }
