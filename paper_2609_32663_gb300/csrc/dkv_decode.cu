@@ -90,6 +90,7 @@ __device__ __forceinline__ void bf8_to_f2x4(const uint4& w, uint64_t* out)
 template <int G_, int LPR_, int TR_, int NS_, int NW_>
 struct PK {
     static constexpr int G = G_, LPR = LPR_, TR = TR_, NS = NS_, NW = NW_;
+    static_assert(PRE <= NS, "the tiles fetched before the PDL wait fit the warp's ring");
     static constexpr int RPS = 32 / LPR;
     static constexpr int DPL = kHeadDim / LPR;
     static constexpr int NCH = DPL / 8;

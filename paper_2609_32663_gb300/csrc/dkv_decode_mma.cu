@@ -39,6 +39,7 @@ template <int G_, int NT_, int NS_, int NW_>
 struct MK {
     static constexpr int G = G_, NT = NT_, NS = NS_, NW = NW_, TR = kMmaTR;
     static constexpr int kStageBytes = kMmaStage;
+    static_assert(PRE <= NS, "the tiles fetched before the PDL wait fit the warp's ring");
     static constexpr int kWarpRing = NS * kStageBytes;
     static constexpr int kRingBytes = NW * kWarpRing;
     static constexpr int kBarBytes = NW * NS * 8;
